@@ -1,0 +1,158 @@
+"""Seeded synthetic inputs for the DendSN layer (forward + BPTT backward).
+
+This module only draws random tensors with the shapes and value distributions of
+the layer workloads; it holds none of the neuron's arithmetic. Both the CUDA path
+and the CPU oracle are fed from it, so they see identical bits.
+
+Layout (the library's ABI):
+  x      [T, B, N, K]   branch/compartment input currents, K innermost
+  alpha  [C, K]         compartment decay factors           (Eq. methods-compartment)
+  xi     [C, K]         translation factors                 (Eq. methods-branch-aggregation)
+  zeta   [C, Kb]        dilation factors, Kb = K / G        (Eq. methods-branch-aggregation)
+  kappa  [C, Kb]        branch strengths                    (Eq. methods-soma-input)
+  mask   [C, Kb] or [N, Kb] uint8 branch-gating mask        (Eq. methods-dbg-mask / -sampling)
+  gs     [T, B, N]      upstream gradient w.r.t. the spikes
+  gv     [T, B, N]      upstream gradient w.r.t. the somatic potential (optional)
+
+Neuron n of a sample belongs to parameter channel c(n) = (n // inner) % C, so
+neurons at the spatial positions of one conv channel share a parameter set
+(Methods, "Dendritic spiking neural networks", constraint 3).
+
+Draw order is fixed: x, alpha, xi, zeta, kappa, mask, gs, gv, all from one
+torch.Generator seeded with the workload's seed.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Optional
+
+import torch
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    name: str
+    T: int
+    B: int
+    N: int
+    K: int
+    G: int
+    C: int
+    inner: int
+    dtype: str          # "f32" or "bf16": dtype of x, spikes, gs and gx
+    psi: str            # "mh" (Mexican hat, Eq. methods-mexican-hat) or "identity"
+    reset: str          # "hard" (Eq. methods-lif-reset-charge) or "soft"
+    theta: float = 1.0
+    beta: float = 0.5
+    x_mean: float = 0.3
+    x_std: float = 1.0
+    x_density: float = 1.0        # fraction of nonzero inputs (event-stream layer: 0.2)
+    mask_p: Optional[float] = None  # Bernoulli(p) branch mask; None = no mask
+    mask_per_neuron: bool = False
+    stateless: bool = False
+    residual: bool = False
+    detach_reset: bool = False
+    seed: int = 0
+
+    @property
+    def Kb(self) -> int:
+        return self.K // self.G
+
+    @property
+    def neurons(self) -> int:
+        return self.B * self.N
+
+    @property
+    def neuron_steps(self) -> int:
+        return self.T * self.B * self.N
+
+    @property
+    def x_bytes(self) -> int:
+        return 2 if self.dtype == "bf16" else 4
+
+    def algorithmic_bytes(self) -> dict:
+        """Bytes a fused forward+backward must move per step, by kernel.
+
+        forward : read x (K elements) + write spikes (1 element) per neuron-step
+        backward: re-read x (K) + read gs (1) + write gx (K) per neuron-step
+        Parameters and the mask (< 1 MB, cache-resident) are not counted.
+        """
+        ns, s = self.neuron_steps, self.x_bytes
+        fwd = ns * (self.K * s + s)
+        bwd = ns * (self.K * s + s + self.K * s)
+        return {"forward": fwd, "backward": bwd, "total": fwd + bwd}
+
+    def with_(self, **kw) -> "Workload":
+        return dataclasses.replace(self, **kw)
+
+
+# The five layer shapes: a tiny case, a conv layer, a deeper bf16 conv layer, a
+# long-horizon event-stream layer with sparse input, and a transformer-token layer
+# with per-neuron branch gating.
+WORKLOADS = {
+    "tiny": Workload("tiny", T=4, B=2, N=64, K=4, G=1, C=64, inner=1, dtype="f32",
+                     psi="mh", reset="hard", seed=0),
+    "conv": Workload("conv", T=4, B=64, N=131072, K=4, G=1, C=128, inner=1024,
+                     dtype="f32", psi="mh", reset="hard", seed=1),
+    "deepconv_bf16": Workload("deepconv_bf16", T=8, B=128, N=65536, K=8, G=1, C=256,
+                              inner=256, dtype="bf16", psi="mh", reset="soft", seed=2),
+    "event": Workload("event", T=64, B=32, N=131072, K=4, G=1, C=128, inner=1024,
+                      dtype="f32", psi="mh", reset="hard", x_mean=0.8, x_std=1.0,
+                      x_density=0.2, seed=3),
+    "token_dbg": Workload("token_dbg", T=4, B=64, N=196 * 384, K=8, G=1, C=384, inner=1,
+                          dtype="f32", psi="mh", reset="hard", mask_p=0.5,
+                          mask_per_neuron=True, seed=4),
+}
+
+
+def torch_dtype(w: Workload) -> torch.dtype:
+    return torch.bfloat16 if w.dtype == "bf16" else torch.float32
+
+
+def make_inputs(w: Workload, device: str = "cpu", with_gv: bool = False) -> dict:
+    """Draw every input of one forward+backward step of workload `w`.
+
+    Value distributions: x ~ N(x_mean, x_std) (times Bernoulli(x_density) when
+    sparse), alpha ~ U(0.5, 0.95), xi ~ N(0, 0.1), zeta ~ U(0.8, 1.2),
+    kappa ~ N(1/K, 0.1), mask ~ Bernoulli(mask_p), gs ~ N(0, 1), gv ~ N(0, 1).
+    x, gs are rounded to the workload dtype; parameters stay float32.
+    """
+    g = torch.Generator(device=device)
+    g.manual_seed(w.seed)
+    f32 = dict(dtype=torch.float32, device=device)
+    T, B, N, K, C, Kb = w.T, w.B, w.N, w.K, w.C, w.Kb
+    x = torch.randn((T, B, N, K), generator=g, **f32).mul_(w.x_std).add_(w.x_mean)
+    if w.x_density < 1.0:
+        keep = torch.rand((T, B, N, K), generator=g, **f32) < w.x_density
+        x.mul_(keep)
+        del keep
+    x = x.to(torch_dtype(w))
+    alpha = torch.rand((C, K), generator=g, **f32).mul_(0.45).add_(0.5)
+    xi = torch.randn((C, K), generator=g, **f32).mul_(0.1)
+    zeta = torch.rand((C, Kb), generator=g, **f32).mul_(0.4).add_(0.8)
+    kappa = torch.randn((C, Kb), generator=g, **f32).mul_(0.1).add_(1.0 / K)
+    mask = None
+    if w.mask_p is not None:
+        rows = N if w.mask_per_neuron else C
+        mask = (torch.rand((rows, Kb), generator=g, **f32) < w.mask_p).to(torch.uint8)
+    gs = torch.randn((T, B, N), generator=g, **f32).to(torch_dtype(w))
+    gv = torch.randn((T, B, N), generator=g, **f32) if with_gv else None
+    return dict(x=x, alpha=alpha, xi=xi, zeta=zeta, kappa=kappa, mask=mask, gs=gs, gv=gv)
+
+
+def scaled(w: Workload, B: Optional[int] = None, N: Optional[int] = None,
+           T: Optional[int] = None) -> Workload:
+    """Same layer kind at a smaller size (for oracle-sized parity runs).
+
+    N must stay a multiple of C * inner so the channel map is unchanged.
+    """
+    kw = {}
+    if B is not None:
+        kw["B"] = B
+    if N is not None:
+        if N % (w.C * w.inner) != 0:
+            raise ValueError("N must be a multiple of C*inner")
+        kw["N"] = N
+    if T is not None:
+        kw["T"] = T
+    return w.with_(**kw)
