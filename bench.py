@@ -1,0 +1,451 @@
+#!/usr/bin/env python
+"""Throughput of the fused DendSN layer step (forward + BPTT backward) on GB300.
+
+One step = dendsn_forward + dendsn_backward over one batch of the workload (all of
+x read, spikes written, grad_x and the four parameter gradients produced); with N
+ranks (torchrun) every rank processes its own batch and the parameter gradients
+are summed with one all-reduce (weak scaling).
+
+Prints ONE JSON line on rank 0. Everything else goes to stderr.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload conv] [--impl ours|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "DendSN fwd+bwd neuron-timesteps/sec and achieved HBM GB/s vs 8 TB/s (1 GB300)"
+UNIT = "neuron-steps/s"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+L2_BYTES = 129 * 2**20
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="conv")
+    ap.add_argument("--psi", choices=["mh", "identity"], default=None)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def measured_hbm_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi clock/throttle samples with GPU timestamps, filtered to a window."""
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.out = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=self.out, stderr=subprocess.DEVNULL)
+        except FileNotFoundError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        self.out.flush()
+        self.out.seek(0)
+        rows = []
+        for line in self.out.read().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 10:
+                continue
+            try:
+                ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S")) + \
+                    float("0." + parts[0].split(".")[1]) if "." in parts[0] else 0.0
+                rows.append(dict(t=ts, sm=float(parts[2]), sm_max=float(parts[3]),
+                                 power=float(parts[4]) if parts[4] not in ("[N/A]", "N/A") else None,
+                                 reasons={"hw_slowdown": parts[6], "hw_thermal_slowdown": parts[7],
+                                          "sw_thermal_slowdown": parts[8],
+                                          "sw_power_cap": parts[9]}))
+            except (ValueError, IndexError):
+                continue
+        os.unlink(self.out.name)
+        return rows
+
+    @staticmethod
+    def summarize(rows, t0, t1):
+        win = [r for r in rows if t0 - 0.1 <= r["t"] <= t1 + 0.1]
+        note = "samples inside the timed region"
+        if not win:
+            load = [r for r in rows if r["sm"] > 0.5 * r["sm_max"]]
+            win = load or rows
+            note = "timed region shorter than the sampling period: samples from the loaded run"
+        if not win:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0,
+                    "note": "nvidia-smi unavailable"}
+        reasons = sorted({k for r in win for k, v in r["reasons"].items() if v == "Active"})
+        return {"sm_mhz": statistics.median(r["sm"] for r in win),
+                "sm_max_mhz": max(r["sm_max"] for r in win), "reasons": reasons,
+                "samples": len(win), "note": note}
+
+
+# ------------------------------------------------------------------ traffic record
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2412_06355_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    ent = rec.get(workload, {}).get(kernel)
+    if not ent or ent.get("source_hash") != kernel_source_hash():
+        return None
+    return ent.get("dram_bytes_per_launch")
+
+
+# ------------------------------------------------------------------ oracle (CPU baseline)
+def oracle_sample_rate(w, inp_cpu_fn, target_s: float):
+    """Times the float64 oracle (forward + backward) on a bounded sample of neurons.
+
+    Returns (neuron-steps/s, description of the sample, neuron-steps timed)."""
+    import numpy as np
+    import oracle
+    oracle.build()
+    ocfg = oracle.OracleConfig(T=w.T, K=w.K, G=w.G, C=w.C, psi=w.psi, reset=w.reset,
+                               theta=w.theta, beta=w.beta, stateless=w.stateless,
+                               residual=w.residual, detach_reset=w.detach_reset)
+
+    def run(M):
+        x, chan, mrow, prm, mask, gs = inp_cpu_fn(M)
+        t = time.perf_counter()
+        oracle.forward(ocfg, x, chan, mrow, *prm, mask)
+        oracle.backward(ocfg, x, chan, mrow, *prm, mask, gs)
+        return time.perf_counter() - t
+
+    M = 256
+    dt = run(M)
+    while dt < 0.5 and M < w.B * w.N:
+        M = min(M * 4, w.B * w.N)
+        dt = run(M)
+    M = int(min(w.B * w.N, max(1, M * target_s / max(dt, 1e-6))))
+    dt = run(M)
+    ns = M * w.T
+    return ns / dt, f"{M} neurons x T={w.T} of the workload (forward + backward), 1 thread", ns, dt
+
+
+def cpu_inputs_from(w, inp):
+    """Sampler of M neurons of the device-resident inputs, as host arrays for the oracle."""
+    import numpy as np
+    import torch
+
+    def fn(M):
+        M = min(M, w.B * w.N)
+        flat = torch.arange(M, device=inp["x"].device) * ((w.B * w.N) // M)
+        b, n = flat // w.N, flat % w.N
+        x = inp["x"][:, b, n, :].cpu()
+        gs = inp["gs"][:, b, n].cpu()
+        nn = n.cpu().numpy()
+        chan = ((nn // w.inner) % w.C).astype(np.int32)
+        mrow = (nn if w.mask_per_neuron else chan).astype(np.int32)
+        prm = [inp[k].cpu() for k in ("alpha", "xi", "zeta", "kappa")]
+        mask = None if inp["mask"] is None else inp["mask"].cpu()
+        return x, chan, mrow, prm, mask, gs
+    return fn
+
+
+# ------------------------------------------------------------------ arms
+def workload_of(args):
+    from paper_2412_06355_gb300.workloads import WORKLOADS
+    w = WORKLOADS[args.workload]
+    if args.psi:
+        w = w.with_(psi=args.psi)
+    return w
+
+
+def config_dict(w, extra=None):
+    d = {"workload": w.name, "T": w.T, "B": w.B, "N": w.N, "K": w.K, "G": w.G, "C": w.C,
+         "inner": w.inner, "x_dtype": w.dtype, "psi": w.psi, "reset": w.reset,
+         "mask": (None if w.mask_p is None else
+                  f"Bernoulli({w.mask_p}) per {'neuron' if w.mask_per_neuron else 'channel'}"),
+         "x_density": w.x_density}
+    if extra:
+        d.update(extra)
+    return d
+
+
+def slice_workload(w, M):
+    """The same layer kind with about M neurons (neurons are independent: the
+    per-neuron work is unchanged). Whole rows of C*inner neurons are kept; below one
+    row the channel count shrinks."""
+    P = w.C * w.inner
+    if M >= P:
+        rows = max(1, min(M // P, w.N // P))
+        return w.with_(B=1, N=rows * P)
+    c = max(1, M // w.inner)
+    return w.with_(B=1, C=c, N=c * w.inner)
+
+
+def run_reference(args):
+    """The oracle, as it stands, on the host cores: the slow baseline arm."""
+    if int(os.environ.get("RANK", "0")) != 0:
+        return
+    import oracle
+    from paper_2412_06355_gb300 import workloads
+    oracle.build()
+    w = workload_of(args)
+
+    def one_step(ws, inp):
+        oracle.forward_layer(ws, inp)
+        oracle.backward_layer(ws, inp)
+
+    # size one step to about 90 s / (steps + warmup), between 0.2 s and 2 s
+    per_step = max(0.2, min(2.0, 90.0 / max(args.steps + args.warmup, 1)))
+    probe = slice_workload(w, 4096)
+    pin = workloads.make_inputs(probe, "cpu")
+    t = time.perf_counter()
+    one_step(probe, pin)
+    rate = probe.neuron_steps / max(time.perf_counter() - t, 1e-6)
+    ws = slice_workload(w, int(rate * per_step / w.T))
+    inp = workloads.make_inputs(ws, "cpu")
+    for _ in range(args.warmup):
+        one_step(ws, inp)
+    t = time.perf_counter()
+    for _ in range(args.steps):
+        one_step(ws, inp)
+    dt = time.perf_counter() - t
+    value = args.steps * ws.neuron_steps / dt
+    sample = (f"{ws.B * ws.N} neurons x T={w.T} per step ({ws.C} channels x {ws.inner}; a "
+              f"slice of the {w.name} layer), float64 forward + backward, 1 thread")
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * dt / max(args.steps, 1), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "impl": "reference",
+            "config": config_dict(w, {"sample_neurons_per_step": ws.B * ws.N}),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2412_06355_gb300 import binding, workloads
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    w = workload_of(args)
+    w_rank = w.with_(seed=w.seed + 1000 * rank)
+    binding.load()
+    cfg = binding.config_of(w)
+    inp = workloads.make_inputs(w_rank, str(dev))
+    x, gs = inp["x"], inp["gs"]
+    alpha, xi, zeta, kappa, mask = (inp[k] for k in ("alpha", "xi", "zeta", "kappa", "mask"))
+    saved, scratch = binding.workspace(cfg, dev)
+    spikes = torch.empty(x.shape[:3], dtype=x.dtype, device=dev)
+    gx = torch.empty_like(x)
+    grads = torch.empty(2 * w.C * w.K + 2 * w.C * w.Kb, dtype=torch.float32, device=dev)
+    ga, gxi, gz, gk = torch.split(grads, [w.C * w.K, w.C * w.K, w.C * w.Kb, w.C * w.Kb])
+    stream = torch.cuda.current_stream()
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        binding.dendsn_forward(cfg, x, alpha, xi, zeta, kappa, mask, spikes, None, saved, stream)
+        if ev is not None:
+            ev[1].record(stream)
+        binding.dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, gs, None, saved, gx,
+                                ga, gxi, gz, gk, scratch, stream)
+        if ev is not None:
+            ev[2].record(stream)
+        if world > 1:
+            dist.all_reduce(grads)
+
+    clocks = ClockSampler(dev.index)
+    if rank == 0:
+        clocks.start()
+    for _ in range(args.warmup):
+        step()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    n_launch0 = binding.launch_count()
+    t0 = time.time()
+    start.record(stream)
+    for i in range(args.steps):
+        step(ev[i])
+    end.record(stream)
+    torch.cuda.synchronize()
+    t1 = time.time()
+    n_launch = binding.launch_count() - n_launch0
+    if world > 1:
+        dist.barrier()
+    ms = start.elapsed_time(end)
+    fwd_ms = [e[0].elapsed_time(e[1]) for e in ev]
+    bwd_ms = [e[1].elapsed_time(e[2]) for e in ev]
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    clock = ClockSampler.summarize(clocks.stop(), t0, t1) if rank == 0 else None
+
+    # ---- end to end through the public API, host buffers, copies inside the timed region
+    e2e = None
+    if not args.no_e2e:
+        x_h = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
+        gs_h = torch.empty(gs.shape, dtype=gs.dtype, pin_memory=True)
+        x_h.copy_(x)
+        gs_h.copy_(gs)
+        s_h = torch.empty(spikes.shape, dtype=spikes.dtype, pin_memory=True)
+        gx_h = torch.empty(gx.shape, dtype=gx.dtype, pin_memory=True)
+        g_h = torch.empty(grads.shape, dtype=grads.dtype, pin_memory=True)
+        h2d = x_h.numel() * x_h.element_size() + gs_h.numel() * gs_h.element_size()
+        d2h = (s_h.numel() * s_h.element_size() + gx_h.numel() * gx_h.element_size() +
+               g_h.numel() * g_h.element_size())
+
+        def e2e_step():
+            x.copy_(x_h, non_blocking=True)
+            gs.copy_(gs_h, non_blocking=True)
+            step()
+            s_h.copy_(spikes, non_blocking=True)
+            gx_h.copy_(gx, non_blocking=True)
+            g_h.copy_(grads, non_blocking=True)
+
+        ke = max(3, min(args.steps, 20))
+        for _ in range(3):
+            e2e_step()
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(ke):
+            e2e_step()
+        s1.record(stream)
+        torch.cuda.synchronize()
+        ems = s0.elapsed_time(s1)
+        if world > 1:
+            t = torch.tensor([ems], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ems = float(t.item())
+        e2e = {"value": world * ke * w.neuron_steps / (ems / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": ke}
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    # ---- roofline of the dominant kernel
+    ab = w.algorithmic_bytes()
+    fwd_avg, bwd_avg = statistics.mean(fwd_ms), statistics.mean(bwd_ms)
+    peak, peak_kind = measured_hbm_peak()
+    if bwd_avg >= fwd_avg:
+        kname, kbytes, kms = "dendsn_backward_kernel", ab["backward"], bwd_avg
+    else:
+        kname, kbytes, kms = "dendsn_forward_kernel", ab["forward"], fwd_avg
+    achieved = kbytes / (kms / 1e3) / 1e9
+    step_ms = ms / args.steps
+    value = world * w.neuron_steps / (step_ms / 1e3)
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        rate, sample, _, dt = oracle_sample_rate(w, cpu_inputs_from(w, inp), args.cpu_seconds)
+        cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": sample + f", {dt:.1f} s", "host_cpus": os.cpu_count()}
+    x_bytes = x.numel() * x.element_size()
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": config_dict(w, {
+            "l2": f"inputs larger than L2: x is {x_bytes / 2**20:.0f} MiB per step "
+                  f"(L2 {L2_BYTES // 2**20} MiB), no flush",
+            "parallelism": f"dp{world}" if world > 1 else "single GPU"}),
+        "roofline": {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peak,
+                     "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+                     "traffic": recorded_traffic(kname, w.name),
+                     "algorithmic_bytes_per_launch": kbytes, "avg_launch_ms": kms},
+        "hbm": {"algorithmic_bytes_per_step": ab["total"],
+                "step_gbs": ab["total"] / (step_ms / 1e3) / 1e9,
+                "frac_of_8tbs": ab["total"] / (step_ms / 1e3) / 1e9 / NOMINAL_HBM_GBS,
+                "frac_of_measured": ab["total"] / (step_ms / 1e3) / 1e9 / peak,
+                "forward_ms": fwd_avg, "backward_ms": bwd_avg},
+        "clocks": clock,
+        "e2e": e2e,
+        "gpu_launches": n_launch,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,149 @@
+/*
+ * dendsn.h - C ABI of libdendsn, the fused DendSN layer for NVIDIA GB300 (sm_103a).
+ *
+ * One DendSN layer (arXiv 2412.06355, Methods "Dendritic spiking neuron") maps the
+ * branch input currents X[t, b, n, i] of B samples x N neurons x K compartments
+ * over T time steps to somatic spikes S[t, b, n]:
+ *
+ *   V^d_i[t] = alpha_i V^d_i[t-1] + X_i[t]                 Eq. methods-compartment
+ *   Y_j[t]   = psi( || (V^d_{C_j}[t] - xi_{C_j}) / zeta_j ||_2 )
+ *                                                           Eq. methods-branch-aggregation
+ *   psi(x)   = (1 - x^2) exp(-x^2 / 2)   or   psi(x) = x    Eq. methods-mexican-hat
+ *   Z[t]     = sum_j kappa_j m_j Y_j[t]                     Eq. methods-soma-input,
+ *                                                           Eq. methods-dbg-mask
+ *   V^s[t]   = beta (1 - S[t-1]) V^s[t-1] + Z[t]            Eq. methods-lif-reset-charge
+ *   S[t]     = Theta(V^s[t] - theta)                        Eq. methods-lif-fire
+ *
+ * and its backward is BPTT with the arctan surrogate dS/dV ~ 1/(1 + pi^2 (V - theta)^2)
+ * (Eq. methods-sg). Branch j holds the G consecutive compartments j*G .. j*G+G-1
+ * (G = P/B in the paper's notation); Kb = K / G branches.
+ *
+ * Conventions shared by every entry point
+ *  - All tensor pointers are DEVICE pointers owned by the caller; the library never
+ *    allocates, frees or copies between host and device.
+ *  - Every call is asynchronous on the CUDA stream passed as `stream` (a
+ *    cudaStream_t; NULL = legacy default stream). Argument errors are detected on
+ *    the host before any launch and return a non-zero status with nothing enqueued.
+ *    A failed launch returns DENDSN_ERR_CUDA. dendsn_last_error() describes the most
+ *    recent failure of the calling thread.
+ *  - Layouts are dense row-major:
+ *      x, grad_x            [T, B, N, K]   dtype x_dtype; base 16-byte aligned
+ *      spikes, grad_spikes  [T, B, N]      dtype x_dtype (spikes are exactly 0 or 1)
+ *      v_out, grad_v        [T, B, N]      float32
+ *      alpha, xi            [C, K]         float32
+ *      zeta, kappa          [C, Kb]        float32 (zeta > 0)
+ *      mask                 [C, Kb] (mask_per_neuron = 0) or [N, Kb] (= 1), uint8 0/1,
+ *                           base 4-byte aligned; NULL = all branches active
+ *      grad_alpha, grad_xi  [C, K]         float32, OVERWRITTEN (not accumulated)
+ *      grad_zeta, grad_kappa[C, Kb]        float32, OVERWRITTEN
+ *    Neuron n of every sample uses parameter channel c(n) = (n / inner) % C, so the
+ *    neurons at the spatial positions of a conv channel share parameters (Methods,
+ *    "Dendritic spiking neural networks", constraint 3). N must be a multiple of
+ *    C * inner. A layer-wide decay alpha (the paper's choice) is passed as a [C, K]
+ *    array of equal values; its gradient is the sum of grad_alpha.
+ *  - Supported: K in {1, 2, 4, 8, 16}; G in {1, 2, 4} with G dividing min(K, 4);
+ *    T >= 0; B * N < 2^31 * C * inner. Others return DENDSN_ERR_UNSUPPORTED.
+ */
+#ifndef DENDSN_H
+#define DENDSN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    DENDSN_OK = 0,
+    DENDSN_ERR_INVALID_ARG = 1,   /* NULL pointer, bad size, bad enum value */
+    DENDSN_ERR_UNSUPPORTED = 2,   /* valid but not compiled in (K, G, surrogate) */
+    DENDSN_ERR_MISALIGNED = 3,    /* a pointer violates its alignment rule */
+    DENDSN_ERR_CUDA = 4           /* a CUDA launch failed; see dendsn_last_error() */
+} dendsn_status;
+
+typedef enum { DENDSN_F32 = 0, DENDSN_BF16 = 1 } dendsn_dtype;
+typedef enum { DENDSN_PSI_IDENTITY = 0, DENDSN_PSI_MEXHAT = 1 } dendsn_psi;
+/* HARD: Eq. methods-lif-reset-charge. SOFT: V^s[t] = beta (V^s[t-1] - theta S[t-1]) + Z[t]. */
+typedef enum { DENDSN_RESET_HARD = 0, DENDSN_RESET_SOFT = 1 } dendsn_reset;
+/* ATAN: Eq. methods-sg, the only surrogate the paper uses. */
+typedef enum { DENDSN_SG_ATAN = 0 } dendsn_surrogate;
+
+typedef struct {
+    int32_t T, B, N;        /* time steps, samples, neurons per sample */
+    int32_t K, G;           /* compartments per neuron, compartments per branch */
+    int32_t C, inner;       /* parameter channels; neurons per channel run */
+    int32_t x_dtype;        /* dendsn_dtype of x, spikes, grad_spikes, grad_x */
+    int32_t psi;            /* dendsn_psi */
+    int32_t reset;          /* dendsn_reset */
+    int32_t surrogate;      /* dendsn_surrogate */
+    float theta;            /* firing threshold (1 in Eq. methods-lif-fire) */
+    float beta;             /* somatic decay, 0 <= beta < 1 */
+    int32_t detach_reset;   /* 1: no gradient through the reset term */
+    int32_t mask_per_neuron;/* 0: mask is [C, Kb]; 1: mask is [N, Kb] */
+    int32_t stateless;      /* 1: Stateless Dendrite, V^d = X (Methods, "Stateless compartment") */
+    int32_t residual;       /* 1: Z += mean_i X_i (Eq. methods-residual) */
+} dendsn_config;
+
+/*
+ * Sizes of the two caller-owned device buffers a forward/backward pair needs.
+ *   saved_bytes  : state checkpoints the forward writes and the backward reads
+ *                  (recompute with checkpointing, Results "Constructing deep
+ *                  DendSNNs"); 0 when T is short enough to recompute from X alone.
+ *                  16-byte aligned. Must outlive the backward.
+ *   scratch_bytes: per-block partial sums of the parameter gradients, used only by
+ *                  dendsn_backward. 16-byte aligned. Contents need no initialisation.
+ * Either output pointer may be NULL.
+ */
+dendsn_status dendsn_workspace_size(const dendsn_config *cfg, size_t *saved_bytes,
+                                    size_t *scratch_bytes);
+
+/*
+ * Fused multi-step forward: compartment scan, L2 branch aggregation, psi, masked
+ * kappa reduction and LIF soma, all T steps in one kernel with the state in
+ * registers.
+ *   x        [T,B,N,K] input currents (read)
+ *   alpha..kappa, mask: parameters as above (read)
+ *   spikes   [T,B,N] output (written)
+ *   v_out    [T,B,N] float32 somatic potential V^s (written), or NULL
+ *   saved    checkpoint buffer of saved_bytes (written), or NULL when no backward
+ *            will follow; ignored when saved_bytes == 0
+ */
+dendsn_status dendsn_forward(const dendsn_config *cfg, const void *x, const float *alpha,
+                             const float *xi, const float *zeta, const float *kappa,
+                             const uint8_t *mask, void *spikes, float *v_out, void *saved,
+                             void *stream);
+
+/*
+ * Fused reverse-time backward (BPTT with the arctan surrogate, Eq. methods-sg). The
+ * forward of each checkpoint interval is recomputed from x in registers.
+ *   grad_spikes [T,B,N] dL/dS (read); grad_v [T,B,N] float32 dL/dV^s (read) or NULL
+ *   saved       the buffer the forward filled (read); may be NULL if saved_bytes == 0
+ *   grad_x      [T,B,N,K] dL/dX (written)
+ *   grad_alpha, grad_xi, grad_zeta, grad_kappa: parameter gradients summed over time,
+ *               samples and the neurons of each channel (written, deterministic order).
+ *               grad_alpha is all zero for a Stateless Dendrite. grad_kappa is the
+ *               gradient w.r.t. the unmasked strength (zero where the mask is 0).
+ *   scratch     scratch_bytes of device memory (contents are overwritten)
+ */
+dendsn_status dendsn_backward(const dendsn_config *cfg, const void *x, const float *alpha,
+                              const float *xi, const float *zeta, const float *kappa,
+                              const uint8_t *mask, const void *grad_spikes,
+                              const float *grad_v, const void *saved, void *grad_x,
+                              float *grad_alpha, float *grad_xi, float *grad_zeta,
+                              float *grad_kappa, void *scratch, void *stream);
+
+/* Static description of a status code. */
+const char *dendsn_status_string(dendsn_status status);
+
+/* Message describing the calling thread's most recent failed call ("" if none). */
+const char *dendsn_last_error(void);
+
+/* Number of kernels the library enqueued since load (all threads). */
+uint64_t dendsn_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DENDSN_H */

@@ -1,0 +1,230 @@
+"""Thin ctypes binding of libdendsn (include/dendsn.h).
+
+Argument marshalling only: every step of the DendSN forward and backward runs in
+the library's CUDA kernels. torch supplies device memory and the current stream.
+There is no fallback: if the library cannot be loaded, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from typing import Optional
+
+import torch
+
+from . import build as _build
+
+F32, BF16 = 0, 1
+PSI_IDENTITY, PSI_MEXHAT = 0, 1
+RESET_HARD, RESET_SOFT = 0, 1
+SG_ATAN = 0
+
+STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported configuration",
+          3: "misaligned pointer", 4: "CUDA error"}
+
+
+class DendSNError(RuntimeError):
+    def __init__(self, fn: str, status: int, msg: str):
+        super().__init__(f"{fn}: {STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+class dendsn_config(ctypes.Structure):
+    """Mirror of the C struct dendsn_config."""
+    _fields_ = [("T", ctypes.c_int32), ("B", ctypes.c_int32), ("N", ctypes.c_int32),
+                ("K", ctypes.c_int32), ("G", ctypes.c_int32), ("C", ctypes.c_int32),
+                ("inner", ctypes.c_int32), ("x_dtype", ctypes.c_int32),
+                ("psi", ctypes.c_int32), ("reset", ctypes.c_int32),
+                ("surrogate", ctypes.c_int32), ("theta", ctypes.c_float),
+                ("beta", ctypes.c_float), ("detach_reset", ctypes.c_int32),
+                ("mask_per_neuron", ctypes.c_int32), ("stateless", ctypes.c_int32),
+                ("residual", ctypes.c_int32)]
+
+    @property
+    def Kb(self) -> int:
+        return self.K // self.G
+
+
+def make_config(T, B, N, K, G=1, C=1, inner=1, dtype="f32", psi="mh", reset="hard",
+                theta=1.0, beta=0.5, detach_reset=False, mask_per_neuron=False,
+                stateless=False, residual=False, surrogate=SG_ATAN) -> dendsn_config:
+    return dendsn_config(T, B, N, K, G, C, inner, BF16 if dtype == "bf16" else F32,
+                         PSI_MEXHAT if psi == "mh" else PSI_IDENTITY,
+                         RESET_SOFT if reset == "soft" else RESET_HARD, surrogate,
+                         float(theta), float(beta), int(detach_reset), int(mask_per_neuron),
+                         int(stateless), int(residual))
+
+
+def config_of(w) -> dendsn_config:
+    """Config of a workloads.Workload."""
+    return make_config(w.T, w.B, w.N, w.K, w.G, w.C, w.inner, w.dtype, w.psi, w.reset,
+                       w.theta, w.beta, w.detach_reset, w.mask_per_neuron, w.stateless,
+                       w.residual)
+
+
+_lib = None
+_lock = threading.Lock()
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load() -> ctypes.CDLL:
+    """Load libdendsn.so, building it first when it is missing or stale."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = _build.build()
+            lib = ctypes.CDLL(path)
+            P, cfgp = ctypes.c_void_p, ctypes.POINTER(dendsn_config)
+            lib.dendsn_workspace_size.argtypes = [cfgp, ctypes.POINTER(ctypes.c_size_t),
+                                                  ctypes.POINTER(ctypes.c_size_t)]
+            lib.dendsn_forward.argtypes = [cfgp] + [P] * 10
+            lib.dendsn_backward.argtypes = [cfgp] + [P] * 16
+            for fn in (lib.dendsn_workspace_size, lib.dendsn_forward, lib.dendsn_backward):
+                fn.restype = ctypes.c_int
+            lib.dendsn_status_string.argtypes = [ctypes.c_int]
+            lib.dendsn_status_string.restype = ctypes.c_char_p
+            lib.dendsn_last_error.argtypes = []
+            lib.dendsn_last_error.restype = ctypes.c_char_p
+            lib.dendsn_launch_count.argtypes = []
+            lib.dendsn_launch_count.restype = ctypes.c_uint64
+            _lib = lib
+    return _lib
+
+
+def _check(fn: str, status: int):
+    if status != 0:
+        raise DendSNError(fn, status, load().dendsn_last_error().decode())
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("DendSN tensors must live on a CUDA device")
+    if not t.is_contiguous():
+        raise ValueError("DendSN tensors must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def launch_count() -> int:
+    """Kernels the library has enqueued since it was loaded."""
+    return int(load().dendsn_launch_count())
+
+
+def dendsn_workspace_size(cfg: dendsn_config):
+    """(saved_bytes, scratch_bytes) for this config."""
+    s, w = ctypes.c_size_t(0), ctypes.c_size_t(0)
+    _check("dendsn_workspace_size",
+           load().dendsn_workspace_size(ctypes.byref(cfg), ctypes.byref(s), ctypes.byref(w)))
+    return int(s.value), int(w.value)
+
+
+def dendsn_forward(cfg, x, alpha, xi, zeta, kappa, mask, spikes, v_out=None, saved=None,
+                   stream=None):
+    _check("dendsn_forward", load().dendsn_forward(
+        ctypes.byref(cfg), _ptr(x), _ptr(alpha), _ptr(xi), _ptr(zeta), _ptr(kappa),
+        _ptr(mask), _ptr(spikes), _ptr(v_out), _ptr(saved), _stream(stream)))
+
+
+def dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved, grad_x,
+                    grad_alpha, grad_xi, grad_zeta, grad_kappa, scratch, stream=None):
+    _check("dendsn_backward", load().dendsn_backward(
+        ctypes.byref(cfg), _ptr(x), _ptr(alpha), _ptr(xi), _ptr(zeta), _ptr(kappa),
+        _ptr(mask), _ptr(grad_spikes), _ptr(grad_v), _ptr(saved), _ptr(grad_x),
+        _ptr(grad_alpha), _ptr(grad_xi), _ptr(grad_zeta), _ptr(grad_kappa), _ptr(scratch),
+        _stream(stream)))
+
+
+# ------------------------------------------------------------------ tensor-level helpers
+def _xdtype(cfg) -> torch.dtype:
+    return torch.bfloat16 if cfg.x_dtype == BF16 else torch.float32
+
+
+def _check_shapes(cfg, x, alpha, xi, zeta, kappa, mask):
+    T, B, N, K, C, Kb = cfg.T, cfg.B, cfg.N, cfg.K, cfg.C, cfg.K // cfg.G
+    if tuple(x.shape) != (T, B, N, K) or x.dtype != _xdtype(cfg):
+        raise ValueError(f"x must be {_xdtype(cfg)} [{T},{B},{N},{K}], got {x.dtype} {tuple(x.shape)}")
+    for name, t, shp in (("alpha", alpha, (C, K)), ("xi", xi, (C, K)), ("zeta", zeta, (C, Kb)),
+                         ("kappa", kappa, (C, Kb))):
+        if tuple(t.shape) != shp or t.dtype != torch.float32:
+            raise ValueError(f"{name} must be float32 {shp}, got {t.dtype} {tuple(t.shape)}")
+    if mask is not None:
+        rows = N if cfg.mask_per_neuron else C
+        if tuple(mask.shape) != (rows, Kb) or mask.dtype != torch.uint8:
+            raise ValueError(f"mask must be uint8 [{rows},{Kb}]")
+
+
+def workspace(cfg, device=None):
+    """Allocates (saved, scratch) byte buffers; None where zero bytes are needed."""
+    sb, wb = dendsn_workspace_size(cfg)
+    dev = device or torch.device("cuda")
+    saved = torch.empty(sb, dtype=torch.uint8, device=dev) if sb else None
+    scratch = torch.empty(max(wb, 16), dtype=torch.uint8, device=dev)
+    return saved, scratch
+
+
+def forward(cfg, x, alpha, xi, zeta, kappa, mask=None, want_v=False, saved=None, stream=None):
+    """Allocating forward. Returns (spikes, v or None)."""
+    _check_shapes(cfg, x, alpha, xi, zeta, kappa, mask)
+    spikes = torch.empty(x.shape[:3], dtype=x.dtype, device=x.device)
+    v = torch.empty(x.shape[:3], dtype=torch.float32, device=x.device) if want_v else None
+    dendsn_forward(cfg, x, alpha, xi, zeta, kappa, mask, spikes, v, saved, stream)
+    return spikes, v
+
+
+def backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v=None, saved=None,
+             scratch=None, stream=None):
+    """Allocating backward. Returns dict gx, galpha, gxi, gzeta, gkappa."""
+    _check_shapes(cfg, x, alpha, xi, zeta, kappa, mask)
+    if scratch is None:
+        _, scratch = workspace(cfg, x.device)
+    dev = x.device
+    C, K, Kb = cfg.C, cfg.K, cfg.K // cfg.G
+    out = dict(gx=torch.empty_like(x),
+               galpha=torch.empty((C, K), dtype=torch.float32, device=dev),
+               gxi=torch.empty((C, K), dtype=torch.float32, device=dev),
+               gzeta=torch.empty((C, Kb), dtype=torch.float32, device=dev),
+               gkappa=torch.empty((C, Kb), dtype=torch.float32, device=dev))
+    dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved,
+                    out["gx"], out["galpha"], out["gxi"], out["gzeta"], out["gkappa"],
+                    scratch, stream)
+    return out
+
+
+class DendSNFunction(torch.autograd.Function):
+    """autograd wrapper: S = DendSN(X; alpha, xi, zeta, kappa) (Eq. dendsn).
+
+    alpha may be a scalar tensor (the paper's layer-wide decay) or [C, K]; its
+    gradient is reduced to its own shape. The mask is a constant.
+    """
+
+    @staticmethod
+    def forward(ctx, x, alpha, xi, zeta, kappa, mask, cfg):
+        a = alpha.expand(cfg.C, cfg.K).contiguous().float()
+        saved, scratch = workspace(cfg, x.device)
+        s, _ = forward(cfg, x.contiguous(), a, xi.contiguous(), zeta.contiguous(),
+                       kappa.contiguous(), mask, saved=saved)
+        ctx.cfg = cfg
+        ctx.alpha_shape = alpha.shape
+        ctx.ws = (saved, scratch)
+        ctx.save_for_backward(x, a, xi, zeta, kappa, mask)
+        return s
+
+    @staticmethod
+    def backward(ctx, gs):
+        x, a, xi, zeta, kappa, mask = ctx.saved_tensors
+        saved, scratch = ctx.ws
+        g = backward(ctx.cfg, x, a, xi, zeta, kappa, mask, gs.contiguous().to(x.dtype),
+                     None, saved, scratch)
+        ga = g["galpha"].sum_to_size(ctx.alpha_shape)
+        return g["gx"], ga, g["gxi"], g["gzeta"], g["gkappa"], None, None

@@ -1,0 +1,353 @@
+// C ABI of libdendsn: argument validation, tiling plan, dispatch to the compiled
+// kernel instances, and the deterministic parameter-gradient finalize kernel.
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "dendsn.h"
+#include "dendsn_types.h"
+
+namespace dendsn {
+
+// Sums the block partials of every channel in a fixed order and writes the four
+// parameter gradients. One thread per (channel, gradient slot).
+__global__ void param_grad_finalize_kernel(const FinArgs F) {
+    const Geometry &g = F.g;
+    const int NP = 2 * g.K + 2 * g.Kb;
+    const int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (w >= (int64_t)g.C * NP) return;
+    const int c = (int)(w / NP);
+    const int q = (int)(w % NP);
+    float sum = 0.f;
+    if (g.O > 0 && g.T > 0) {
+        const int ct_lo = (int)(((int64_t)c * g.inner) / g.TXn);
+        const int ct_hi = (int)((((int64_t)c + 1) * g.inner - 1) / g.TXn);
+        for (int ct = ct_lo; ct <= ct_hi; ++ct) {
+            const int lc = c - (int)(((int64_t)ct * g.TXn) / g.inner);
+            for (int rg = 0; rg < g.nRG; ++rg)
+                sum = __fadd_rn(sum, F.partials[(((int64_t)rg * g.nCT + ct) * g.nch_max + lc) * NP + q]);
+        }
+    }
+    if (q < g.K) F.g_alpha[(int64_t)c * g.K + q] = F.stateless ? 0.f : sum;
+    else if (q < 2 * g.K) F.g_xi[(int64_t)c * g.K + (q - g.K)] = sum;
+    else if (q < 2 * g.K + g.Kb) F.g_zeta[(int64_t)c * g.Kb + (q - 2 * g.K)] = sum;
+    else F.g_kappa[(int64_t)c * g.Kb + (q - 2 * g.K - g.Kb)] = sum;
+}
+
+cudaError_t launch_finalize(const FinArgs &a, cudaStream_t s) {
+    const int64_t n = (int64_t)a.g.C * (2 * a.g.K + 2 * a.g.Kb);
+    const int threads = 256;
+    const int blocks = (int)((n + threads - 1) / threads);
+    param_grad_finalize_kernel<<<blocks, threads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace dendsn
+
+using namespace dendsn;
+
+namespace {
+
+thread_local char g_last_error[512] = "";
+std::atomic<uint64_t> g_launches{0};
+
+dendsn_status fail(dendsn_status st, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_last_error, sizeof g_last_error, fmt, ap);
+    va_end(ap);
+    return st;
+}
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+struct Plan {
+    Geometry g;
+    int blocks;        // forward/backward grid
+    int LPN;
+    size_t saved_bytes, scratch_bytes, ck_vd_bytes;
+    int sx;            // bytes per x element
+};
+
+int sm_count() {
+    static int cached = 0;
+    if (cached == 0) {
+        int dev = 0, n = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess &&
+            cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && n > 0)
+            cached = n;
+        else
+            cached = 152;   // GB300
+    }
+    return cached;
+}
+
+bool is01(int32_t v) { return v == 0 || v == 1; }
+
+dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) {
+    if (cfg == nullptr) return fail(DENDSN_ERR_INVALID_ARG, "cfg is NULL");
+    const dendsn_config &c = *cfg;
+    if (c.T < 0 || c.B < 0 || c.N < 0)
+        return fail(DENDSN_ERR_INVALID_ARG, "negative size (T=%d B=%d N=%d)", c.T, c.B, c.N);
+    if (c.C < 1 || c.inner < 1) return fail(DENDSN_ERR_INVALID_ARG, "C and inner must be >= 1");
+    if (c.K < 1 || c.G < 1 || c.K % c.G != 0)
+        return fail(DENDSN_ERR_INVALID_ARG, "need K >= 1, G >= 1 and G | K (K=%d G=%d)", c.K, c.G);
+    if (!(c.x_dtype == DENDSN_F32 || c.x_dtype == DENDSN_BF16))
+        return fail(DENDSN_ERR_INVALID_ARG, "bad x_dtype %d", c.x_dtype);
+    if (!is01(c.psi) || !is01(c.reset) || !is01(c.detach_reset) || !is01(c.mask_per_neuron) ||
+        !is01(c.stateless) || !is01(c.residual))
+        return fail(DENDSN_ERR_INVALID_ARG, "enum/flag field out of range");
+    if (c.surrogate != DENDSN_SG_ATAN)
+        return fail(c.surrogate < 0 ? DENDSN_ERR_INVALID_ARG : DENDSN_ERR_UNSUPPORTED,
+                    "surrogate %d not available (only the arctan surrogate)", c.surrogate);
+    if (!std::isfinite(c.theta) || !std::isfinite(c.beta))
+        return fail(DENDSN_ERR_INVALID_ARG, "theta and beta must be finite");
+    const bool k_ok = c.K == 1 || c.K == 2 || c.K == 4 || c.K == 8 || c.K == 16;
+    const int KT = c.K < 4 ? c.K : 4;
+    if (!k_ok || KT % c.G != 0)
+        return fail(DENDSN_ERR_UNSUPPORTED, "K=%d G=%d not compiled in", c.K, c.G);
+    const int64_t P = (int64_t)c.C * c.inner;
+    if (P > INT32_MAX) return fail(DENDSN_ERR_UNSUPPORTED, "C*inner too large");
+    if (c.N % P != 0)
+        return fail(DENDSN_ERR_INVALID_ARG, "N=%d must be a multiple of C*inner=%lld", c.N,
+                    (long long)P);
+    const int64_t BN = (int64_t)c.B * c.N;
+    const int64_t O = BN / P;
+    if (O > INT32_MAX) return fail(DENDSN_ERR_UNSUPPORTED, "too many rows");
+
+    Geometry &g = pl->g;
+    std::memset(&g, 0, sizeof g);
+    const int LPN = c.K / KT;
+    const int W = 32 / LPN;                     // columns per warp
+    const int full = kThreads / LPN;            // columns of a one-row tile
+    g.O = O;
+    g.BN = BN;
+    g.P = (int32_t)P;
+    g.N = c.N;
+    g.C = c.C;
+    g.inner = c.inner;
+    g.T = c.T;
+    g.K = c.K;
+    g.Kb = c.K / c.G;
+    g.TXn = (c.inner >= W && P % full == 0) ? full : W;
+    g.TY = kThreads / (g.TXn * LPN);
+    g.seg = (c.inner % W == 0) ? W : ((W % c.inner == 0) ? c.inner : 1);
+    g.nCT = (int32_t)((P + g.TXn - 1) / g.TXn);
+    g.L = (c.T <= 4) ? 4 : 8;
+    g.n_ck = (c.T > g.L) ? (c.T + g.L - 1) / g.L - 1 : 0;
+    // rows per thread: about 16 blocks per SM in total, but at least one row
+    const int64_t target_blocks = 16LL * (need_sm_count ? sm_count() : 152);
+    const int64_t rg_target = std::max<int64_t>(1, (target_blocks + g.nCT - 1) / g.nCT);
+    const int64_t rows_per_rg = std::max<int64_t>(1, (O + rg_target - 1) / rg_target);
+    g.R = (int32_t)std::max<int64_t>(1, (rows_per_rg + g.TY - 1) / g.TY);
+    const int64_t nRG = (O + (int64_t)g.R * g.TY - 1) / ((int64_t)g.R * g.TY);
+    g.nRG = (int32_t)nRG;
+    g.nch_max = std::min<int32_t>(c.C, (g.TXn - 1) / c.inner + 2);
+    const int64_t blocks = (int64_t)g.nCT * nRG;
+    if (blocks > INT32_MAX) return fail(DENDSN_ERR_UNSUPPORTED, "grid too large");
+    pl->blocks = (int)blocks;
+    pl->LPN = LPN;
+    pl->sx = (c.x_dtype == DENDSN_BF16) ? 2 : 4;
+    const size_t NP = 2 * (size_t)c.K + 2 * (size_t)g.Kb;
+    pl->scratch_bytes = (size_t)blocks * g.nch_max * NP * sizeof(float);
+    pl->scratch_bytes = (pl->scratch_bytes + 15) / 16 * 16;
+    pl->ck_vd_bytes = (size_t)g.n_ck * (size_t)BN * c.K * sizeof(float);
+    pl->saved_bytes = pl->ck_vd_bytes + (size_t)g.n_ck * (size_t)BN * sizeof(float);
+    pl->saved_bytes = (pl->saved_bytes + 15) / 16 * 16;
+    return DENDSN_OK;
+}
+
+Params make_params(const dendsn_config &c, const float *alpha, const float *xi,
+                   const float *zeta, const float *kappa, const uint8_t *mask) {
+    Params p;
+    p.alpha = alpha;
+    p.xi = xi;
+    p.zeta = zeta;
+    p.kappa = kappa;
+    p.mask = mask;
+    p.mask_mode = mask == nullptr ? 0 : (c.mask_per_neuron ? 2 : 1);
+    p.theta = c.theta;
+    p.beta = c.beta;
+    p.soft = c.reset == DENDSN_RESET_SOFT;
+    p.stateless = c.stateless;
+    p.residual = c.residual;
+    p.detach = c.detach_reset;
+    return p;
+}
+
+dendsn_status check_params(const float *alpha, const float *xi, const float *zeta,
+                           const float *kappa, const uint8_t *mask) {
+    if (!alpha || !xi || !zeta || !kappa)
+        return fail(DENDSN_ERR_INVALID_ARG, "parameter pointer is NULL");
+    if (!aligned(alpha, 4) || !aligned(xi, 4) || !aligned(zeta, 4) || !aligned(kappa, 4))
+        return fail(DENDSN_ERR_MISALIGNED, "parameters must be 4-byte aligned");
+    if (mask && !aligned(mask, 4)) return fail(DENDSN_ERR_MISALIGNED, "mask must be 4-byte aligned");
+    return DENDSN_OK;
+}
+
+#define DENDSN_FWD_CASE(KK, GG)                                                       \
+    if (cfg.K == KK && cfg.G == GG) {                                                 \
+        switch (cfg.psi * 2 + cfg.x_dtype) {                                        \
+        case 0: return launch_forward<KK, GG, 0, 0>(a, blocks, s);                    \
+        case 1: return launch_forward<KK, GG, 0, 1>(a, blocks, s);                    \
+        case 2: return launch_forward<KK, GG, 1, 0>(a, blocks, s);                    \
+        default: return launch_forward<KK, GG, 1, 1>(a, blocks, s);                   \
+        }                                                                           \
+    }
+
+cudaError_t dispatch_forward(const dendsn_config &cfg, const FwdArgs &a, int blocks,
+                             cudaStream_t s) {
+    DENDSN_KG_LIST(DENDSN_FWD_CASE)
+    return cudaErrorInvalidValue;
+}
+
+#define DENDSN_BWD_CASE(KK, GG)                                                       \
+    if (cfg.K == KK && cfg.G == GG) {                                                 \
+        if (L == 4) {                                                               \
+            switch (cfg.psi * 2 + cfg.x_dtype) {                                    \
+            case 0: return launch_backward<KK, GG, 0, 0, 4>(a, blocks, s);            \
+            case 1: return launch_backward<KK, GG, 0, 1, 4>(a, blocks, s);            \
+            case 2: return launch_backward<KK, GG, 1, 0, 4>(a, blocks, s);            \
+            default: return launch_backward<KK, GG, 1, 1, 4>(a, blocks, s);           \
+            }                                                                       \
+        }                                                                           \
+        switch (cfg.psi * 2 + cfg.x_dtype) {                                        \
+        case 0: return launch_backward<KK, GG, 0, 0, 8>(a, blocks, s);                \
+        case 1: return launch_backward<KK, GG, 0, 1, 8>(a, blocks, s);                \
+        case 2: return launch_backward<KK, GG, 1, 0, 8>(a, blocks, s);                \
+        default: return launch_backward<KK, GG, 1, 1, 8>(a, blocks, s);               \
+        }                                                                           \
+    }
+
+cudaError_t dispatch_backward(const dendsn_config &cfg, int L, const BwdArgs &a, int blocks,
+                              cudaStream_t s) {
+    DENDSN_KG_LIST(DENDSN_BWD_CASE)
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+extern "C" {
+
+dendsn_status dendsn_workspace_size(const dendsn_config *cfg, size_t *saved_bytes,
+                                    size_t *scratch_bytes) {
+    Plan pl;
+    dendsn_status st = make_plan(cfg, &pl, true);
+    if (st != DENDSN_OK) return st;
+    if (saved_bytes) *saved_bytes = pl.saved_bytes;
+    if (scratch_bytes) *scratch_bytes = pl.scratch_bytes;
+    return DENDSN_OK;
+}
+
+dendsn_status dendsn_forward(const dendsn_config *cfg, const void *x, const float *alpha,
+                             const float *xi, const float *zeta, const float *kappa,
+                             const uint8_t *mask, void *spikes, float *v_out, void *saved,
+                             void *stream) {
+    Plan pl;
+    dendsn_status st = make_plan(cfg, &pl, true);
+    if (st != DENDSN_OK) return st;
+    if (pl.g.BN == 0 || pl.g.T == 0) return DENDSN_OK;
+    if (!x || !spikes) return fail(DENDSN_ERR_INVALID_ARG, "x or spikes is NULL");
+    if ((st = check_params(alpha, xi, zeta, kappa, mask)) != DENDSN_OK) return st;
+    if (!aligned(x, 16)) return fail(DENDSN_ERR_MISALIGNED, "x must be 16-byte aligned");
+    if (!aligned(spikes, pl.sx)) return fail(DENDSN_ERR_MISALIGNED, "spikes misaligned");
+    if (v_out && !aligned(v_out, 4)) return fail(DENDSN_ERR_MISALIGNED, "v_out misaligned");
+    if (saved && !aligned(saved, 16)) return fail(DENDSN_ERR_MISALIGNED, "saved must be 16-byte aligned");
+    FwdArgs a;
+    a.g = pl.g;
+    a.p = make_params(*cfg, alpha, xi, zeta, kappa, mask);
+    a.x = x;
+    a.spikes = spikes;
+    a.v_out = v_out;
+    a.ck_vd = (saved && pl.g.n_ck > 0) ? static_cast<float *>(saved) : nullptr;
+    a.ck_vs = a.ck_vd ? reinterpret_cast<float *>(static_cast<char *>(saved) + pl.ck_vd_bytes)
+                      : nullptr;
+    cudaError_t e = dispatch_forward(*cfg, a, pl.blocks, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess)
+        return fail(DENDSN_ERR_CUDA, "forward launch failed: %s", cudaGetErrorString(e));
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    return DENDSN_OK;
+}
+
+dendsn_status dendsn_backward(const dendsn_config *cfg, const void *x, const float *alpha,
+                              const float *xi, const float *zeta, const float *kappa,
+                              const uint8_t *mask, const void *grad_spikes,
+                              const float *grad_v, const void *saved, void *grad_x,
+                              float *grad_alpha, float *grad_xi, float *grad_zeta,
+                              float *grad_kappa, void *scratch, void *stream) {
+    Plan pl;
+    dendsn_status st = make_plan(cfg, &pl, true);
+    if (st != DENDSN_OK) return st;
+    if (!grad_alpha || !grad_xi || !grad_zeta || !grad_kappa)
+        return fail(DENDSN_ERR_INVALID_ARG, "parameter-gradient pointer is NULL");
+    if (!aligned(grad_alpha, 4) || !aligned(grad_xi, 4) || !aligned(grad_zeta, 4) ||
+        !aligned(grad_kappa, 4))
+        return fail(DENDSN_ERR_MISALIGNED, "parameter gradients must be 4-byte aligned");
+    const bool work = pl.g.BN > 0 && pl.g.T > 0;
+    if (work) {
+        if (!x || !grad_spikes || !grad_x)
+            return fail(DENDSN_ERR_INVALID_ARG, "x, grad_spikes or grad_x is NULL");
+        if ((st = check_params(alpha, xi, zeta, kappa, mask)) != DENDSN_OK) return st;
+        if (!aligned(x, 16) || !aligned(grad_x, 16))
+            return fail(DENDSN_ERR_MISALIGNED, "x and grad_x must be 16-byte aligned");
+        if (!aligned(grad_spikes, pl.sx)) return fail(DENDSN_ERR_MISALIGNED, "grad_spikes misaligned");
+        if (grad_v && !aligned(grad_v, 4)) return fail(DENDSN_ERR_MISALIGNED, "grad_v misaligned");
+        if (pl.g.n_ck > 0 && !saved)
+            return fail(DENDSN_ERR_INVALID_ARG, "T=%d needs the forward's saved checkpoints", pl.g.T);
+        if (saved && !aligned(saved, 16)) return fail(DENDSN_ERR_MISALIGNED, "saved must be 16-byte aligned");
+        if (!scratch) return fail(DENDSN_ERR_INVALID_ARG, "scratch is NULL");
+        if (!aligned(scratch, 16)) return fail(DENDSN_ERR_MISALIGNED, "scratch must be 16-byte aligned");
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (work) {
+        BwdArgs a;
+        a.g = pl.g;
+        a.p = make_params(*cfg, alpha, xi, zeta, kappa, mask);
+        a.x = x;
+        a.gs = grad_spikes;
+        a.gv = grad_v;
+        a.ck_vd = pl.g.n_ck > 0 ? static_cast<const float *>(saved) : nullptr;
+        a.ck_vs = pl.g.n_ck > 0 ? reinterpret_cast<const float *>(
+                                      static_cast<const char *>(saved) + pl.ck_vd_bytes)
+                                : nullptr;
+        a.gx = grad_x;
+        a.partials = static_cast<float *>(scratch);
+        cudaError_t e = dispatch_backward(*cfg, pl.g.L, a, pl.blocks, s);
+        if (e != cudaSuccess)
+            return fail(DENDSN_ERR_CUDA, "backward launch failed: %s", cudaGetErrorString(e));
+        g_launches.fetch_add(1, std::memory_order_relaxed);
+    }
+    FinArgs f;
+    f.g = pl.g;
+    f.partials = static_cast<const float *>(scratch);
+    f.g_alpha = grad_alpha;
+    f.g_xi = grad_xi;
+    f.g_zeta = grad_zeta;
+    f.g_kappa = grad_kappa;
+    f.stateless = cfg->stateless;
+    cudaError_t e = launch_finalize(f, s);
+    if (e != cudaSuccess)
+        return fail(DENDSN_ERR_CUDA, "finalize launch failed: %s", cudaGetErrorString(e));
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    return DENDSN_OK;
+}
+
+const char *dendsn_status_string(dendsn_status status) {
+    switch (status) {
+    case DENDSN_OK: return "ok";
+    case DENDSN_ERR_INVALID_ARG: return "invalid argument";
+    case DENDSN_ERR_UNSUPPORTED: return "unsupported configuration";
+    case DENDSN_ERR_MISALIGNED: return "misaligned pointer";
+    case DENDSN_ERR_CUDA: return "CUDA error";
+    }
+    return "unknown status";
+}
+
+const char *dendsn_last_error(void) { return g_last_error; }
+
+uint64_t dendsn_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+}  // extern "C"

@@ -1,0 +1,80 @@
+// Host/device argument blocks and launcher declarations of the DendSN kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace dendsn {
+
+enum { PSI_IDENTITY = 0, PSI_MEXHAT = 1 };
+
+constexpr int kThreads = 256;     // threads per block of the forward/backward kernels
+constexpr int kFwdBatch = 4;      // time steps per load batch in the forward
+
+// Tiling and sizes shared by every kernel of one call (computed on the host).
+// Neuron j = o * P + p: row o in [0, O), column p in [0, P); channel = p / inner.
+struct Geometry {
+    int64_t O;        // rows
+    int64_t BN;       // neurons = O * P
+    int32_t P;        // columns = C * inner
+    int32_t N, C, inner, T;
+    int32_t K, Kb;
+    int32_t TXn, TY;  // block tile: TXn columns x TY row lanes (x LPN lanes per neuron)
+    int32_t R;        // rows per thread
+    int32_t nCT;      // column tiles
+    int32_t nRG;      // row groups (blocks along the rows)
+    int32_t L;        // backward chunk length == checkpoint interval
+    int32_t n_ck;     // checkpoints stored by the forward: ceil(T / L) - 1 when T > L, else 0
+    int32_t nch_max;  // most channels one column tile can touch
+    int32_t seg;      // columns of one warp that share a channel (power of 2)
+};
+
+struct Params {
+    const float *alpha, *xi, *zeta, *kappa;
+    const uint8_t *mask;
+    int32_t mask_mode;   // 0 none, 1 per channel [C,Kb], 2 per neuron [N,Kb]
+    float theta, beta;
+    int32_t soft, stateless, residual, detach;
+};
+
+struct FwdArgs {
+    Geometry g;
+    Params p;
+    const void *x;
+    void *spikes;
+    float *v_out;
+    float *ck_vd;   // [n_ck][BN][K]  or NULL (no checkpoints written)
+    float *ck_vs;   // [n_ck][BN]
+};
+
+struct BwdArgs {
+    Geometry g;
+    Params p;
+    const void *x;
+    const void *gs;
+    const float *gv;
+    const float *ck_vd;
+    const float *ck_vs;
+    void *gx;
+    float *partials;   // [nCT * nRG][nch_max][NP], NP = 2K + 2Kb
+};
+
+struct FinArgs {
+    Geometry g;
+    const float *partials;
+    float *g_alpha, *g_xi, *g_zeta, *g_kappa;
+    int32_t stateless;
+};
+
+// XT: 0 = float, 1 = bfloat16. Defined in the instantiation units.
+template <int K, int G, int PSI, int XT>
+cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s);
+template <int K, int G, int PSI, int XT, int L>
+cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s);
+cudaError_t launch_finalize(const FinArgs &a, cudaStream_t s);
+
+}  // namespace dendsn
+
+// (K, G) pairs compiled into the library: K compartments per neuron, G per branch.
+#define DENDSN_KG_LIST(X) \
+    X(1, 1) X(2, 1) X(2, 2) X(4, 1) X(4, 2) X(4, 4) X(8, 1) X(8, 2) X(8, 4) X(16, 1) X(16, 2) X(16, 4)

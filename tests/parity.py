@@ -1,0 +1,116 @@
+"""Shared machinery of the GPU-vs-oracle parity tests.
+
+Tolerances (written here once, used by every parity test):
+  V^s      |gpu - oracle| <= 1e-6 + 1e-5 |oracle|             (float32 state)
+  spikes   identical, except at and after a step where the oracle's potential lies
+           within 1e-5 of the threshold (an "ambiguous" step: float32 rounding may
+           legitimately decide it either way)
+  grads    |gpu - oracle| <= rtol |oracle| + atol_rel * rms(oracle)
+           float32: rtol 1e-4, atol_rel 1e-5;  bfloat16 grad_x: rtol 2e-2, atol_rel 1e-2
+           parameter gradients (float32 sums over up to 10^6 terms): rtol 1e-4,
+           atol_rel 1e-5
+  atol_rel: an element that is a near-cancelling sum of terms of size ~rms carries
+  an absolute float32 rounding error ~(number of terms) * 6e-8 * rms, so a pure
+  relative bound is meaningless for it; 1e-5 * rms covers sums of up to ~150
+  terms, which bounds the reverse scans here (alpha <= 0.95: weights below 1e-3
+  after 135 steps) and the per-thread parameter sums.
+
+Neurons whose oracle trajectory has an ambiguous step get zero upstream gradient
+(grad_spikes and grad_v) on BOTH sides: the backward is linear in them, so those
+neurons then contribute exactly zero to every gradient whatever spike pattern
+each side followed, and the remaining comparisons stay exact-trajectory ones.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+from paper_2412_06355_gb300 import binding, workloads
+
+AMBIGUOUS = 1e-5
+V_RTOL, V_ATOL = 1e-5, 1e-6
+G_RTOL, G_ATOL_REL = 1e-4, 1e-5
+BF16_RTOL, BF16_ATOL_REL = 2e-2, 1e-2
+
+
+def rms(a: np.ndarray) -> float:
+    return float(np.sqrt(np.mean(np.square(a)))) if a.size else 0.0
+
+
+def assert_close(name, got, want, rtol, atol_rel, mask=None, atol_abs=0.0):
+    got = np.asarray(got, np.float64)
+    want = np.asarray(want, np.float64)
+    assert got.shape == want.shape, (name, got.shape, want.shape)
+    if mask is not None:
+        got, want = got[mask], want[mask]
+    assert np.all(np.isfinite(got)), f"{name}: non-finite values"
+    atol = atol_rel * rms(want) + atol_abs
+    err = np.abs(got - want)
+    bound = rtol * np.abs(want) + atol
+    bad = err > bound
+    if bad.any():
+        i = np.argmax(err - bound)
+        raise AssertionError(
+            f"{name}: {int(bad.sum())}/{bad.size} elements out of tolerance; worst "
+            f"got={got.flat[i]!r} want={want.flat[i]!r} err={err.flat[i]:.3e} "
+            f"bound={bound.flat[i]:.3e} (rtol={rtol}, atol={atol:.3e})")
+
+
+def first_ambiguous_step(v_oracle: np.ndarray, theta: float) -> np.ndarray:
+    """Per neuron ([T, ...] input): index of the first ambiguous step, or T."""
+    amb = np.abs(v_oracle - theta) < AMBIGUOUS
+    T = v_oracle.shape[0]
+    first = np.where(amb.any(axis=0), amb.argmax(axis=0), T)
+    return first
+
+
+def to_dev(inp: dict, device="cuda") -> dict:
+    return {k: (None if v is None else v.to(device).contiguous()) for k, v in inp.items()}
+
+
+def run_gpu(w, inp_dev: dict, gs, gv, want_v=True):
+    """Forward + backward through the C ABI; returns host numpy results."""
+    cfg = binding.config_of(w)
+    saved, scratch = binding.workspace(cfg)
+    s, v = binding.forward(cfg, inp_dev["x"], inp_dev["alpha"], inp_dev["xi"],
+                           inp_dev["zeta"], inp_dev["kappa"], inp_dev["mask"], want_v=want_v,
+                           saved=saved)
+    g = binding.backward(cfg, inp_dev["x"], inp_dev["alpha"], inp_dev["xi"], inp_dev["zeta"],
+                         inp_dev["kappa"], inp_dev["mask"], gs, gv, saved, scratch)
+    torch.cuda.synchronize()
+    out = {"s": oracle.to_f64(s), "v": None if v is None else oracle.to_f64(v)}
+    out.update({k: oracle.to_f64(t) for k, t in g.items()})
+    return out
+
+
+def check_layer(w, seed_inputs=None, with_gv=True):
+    """Full parity check of workload `w` (all neurons) against the oracle."""
+    inp = seed_inputs if seed_inputs is not None else workloads.make_inputs(w, "cpu", with_gv=with_gv)
+    s_o, v_o = oracle.forward_layer(w, inp)
+    first = first_ambiguous_step(v_o, w.theta)              # [B, N]
+    amb = first < w.T
+    gs = inp["gs"].clone()
+    gs[:, torch.from_numpy(amb)] = 0
+    gv = None
+    if inp.get("gv") is not None:
+        gv = inp["gv"].clone()
+        gv[:, torch.from_numpy(amb)] = 0
+    dev = to_dev(inp)
+    got = run_gpu(w, dev, gs.cuda(), None if gv is None else gv.cuda())
+    ref = oracle.backward_layer(w, dict(inp, gv=gv), gs=gs)
+
+    t_idx = np.arange(w.T)[:, None, None]
+    v_mask = t_idx <= first[None]                           # V compared up to the first ambiguous step
+    s_mask = t_idx < first[None]                            # S compared before it
+    assert_close("V^s", got["v"], v_o, V_RTOL, 0.0, mask=v_mask, atol_abs=V_ATOL)
+    assert np.array_equal(got["s"][s_mask], s_o[s_mask]), \
+        f"spikes differ at {int((got['s'][s_mask] != s_o[s_mask]).sum())} unambiguous steps"
+    assert set(np.unique(got["s"]).tolist()) <= {0.0, 1.0}
+    if w.dtype == "bf16":
+        assert_close("grad_x", got["gx"], ref["gx"], BF16_RTOL, BF16_ATOL_REL)
+    else:
+        assert_close("grad_x", got["gx"], ref["gx"], G_RTOL, G_ATOL_REL)
+    for k in ("galpha", "gxi", "gzeta", "gkappa"):
+        assert_close(k, got[k], ref[k], G_RTOL, G_ATOL_REL)
+    return dict(ambiguous_neurons=int(amb.sum()), spikes=float(s_o.mean()))

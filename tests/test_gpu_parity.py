@@ -1,0 +1,225 @@
+"""GPU parity: the CUDA path through the C ABI against the float64 oracle.
+
+Tolerances and the handling of threshold-ambiguous steps are in tests/parity.py.
+* every layer workload at a size the oracle finishes in seconds (all neurons),
+  with both branch nonlinearities;
+* edge cases: every compiled (K, G), ragged tiles and chunks, T = 0 / 1,
+  empty batch, every flag, extreme threshold/decay;
+* the full-size workloads in the benchmark's launch configuration, compared on a
+  sample of neurons (neurons are independent), with parameter gradients checked
+  by giving the non-sampled neurons zero upstream gradient (the backward is
+  linear in it, so the sums then run over the sample only).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2412_06355_gb300 import binding, workloads
+from paper_2412_06355_gb300.workloads import WORKLOADS, scaled
+
+from parity import (BF16_ATOL_REL, BF16_RTOL, G_ATOL_REL, G_RTOL, V_ATOL, V_RTOL,
+                    assert_close, check_layer, first_ambiguous_step, to_dev)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.fail("these tests need a CUDA device")
+    binding.load()
+    oracle.build()
+
+
+SCALED = {
+    "tiny": WORKLOADS["tiny"],
+    "conv": scaled(WORKLOADS["conv"], B=2),
+    "deepconv_bf16": scaled(WORKLOADS["deepconv_bf16"], B=2),
+    "event": WORKLOADS["event"].with_(C=32, N=32 * 1024, B=2),
+    "token_dbg": scaled(WORKLOADS["token_dbg"], B=2),
+}
+
+
+@pytest.mark.parametrize("psi", ["mh", "identity"])
+@pytest.mark.parametrize("name", list(SCALED))
+def test_layer_workloads(name, psi):
+    w = SCALED[name].with_(psi=psi)
+    info = check_layer(w)
+    assert info["spikes"] > 0.0
+
+
+KG = [(1, 1), (2, 1), (2, 2), (4, 1), (4, 2), (4, 4), (8, 1), (8, 2), (8, 4),
+      (16, 1), (16, 2), (16, 4)]
+
+
+@pytest.mark.parametrize("K,G", KG)
+def test_every_compiled_kg(K, G):
+    i = KG.index((K, G))
+    w = workloads.Workload(
+        f"kg{K}_{G}", T=9, B=3, N=35 * 2, K=K, G=G, C=5, inner=7,
+        dtype="bf16" if i % 3 == 2 else "f32", psi="mh" if i % 2 == 0 else "identity",
+        reset="soft" if i % 4 == 1 else "hard", mask_p=0.6 if i % 2 else None,
+        mask_per_neuron=(i % 4 == 3), seed=100 + i)
+    check_layer(w)
+
+
+@pytest.mark.parametrize("kw", [
+    dict(stateless=True), dict(residual=True), dict(stateless=True, residual=True),
+    dict(detach_reset=True), dict(detach_reset=True, reset="soft"),
+    dict(reset="soft", psi="identity"), dict(theta=0.0), dict(beta=0.0),
+    dict(theta=0.25, beta=0.95), dict(mask_p=0.5), dict(mask_p=0.5, mask_per_neuron=True),
+    dict(mask_p=0.0),
+], ids=lambda kw: "-".join(f"{k}={v}" for k, v in kw.items()))
+def test_variants(kw):
+    w = workloads.Workload("var", T=6, B=4, N=4 * 96, K=8, G=1, C=4, inner=96, dtype="f32",
+                           psi="mh", reset="hard", seed=7).with_(**kw)
+    check_layer(w)
+
+
+@pytest.mark.parametrize("T", [1, 2, 3, 5, 8, 9, 16, 17, 64, 70])
+def test_time_lengths_and_checkpoint_chunks(T):
+    w = workloads.Workload("t", T=T, B=3, N=2 * 160, K=4, G=2, C=2, inner=160, dtype="f32",
+                           psi="identity" if T % 2 else "mh", reset="hard" if T % 3 else "soft",
+                           x_mean=0.5, seed=T)
+    check_layer(w)
+
+
+def test_ragged_column_tiles_and_odd_inner():
+    # P = C*inner = 300: not a multiple of any tile width; inner = 100 is not a power of 2
+    w = workloads.Workload("ragged", T=5, B=3, N=600, K=4, G=1, C=3, inner=100, dtype="f32",
+                           psi="mh", reset="hard", seed=9)
+    check_layer(w)
+    w = w.with_(K=8, dtype="bf16", inner=50, N=300, seed=10)
+    check_layer(w)
+
+
+def test_large_inner_and_sparse_zero_inputs():
+    # exact zeros with xi = 0 hit r_b = 0 (subgradient 0) for the identity branch
+    w = workloads.Workload("zeros", T=12, B=2, N=2048, K=4, G=2, C=2, inner=1024, dtype="f32",
+                           psi="identity", reset="hard", x_mean=0.8, x_density=0.2, seed=12)
+    inp = workloads.make_inputs(w, "cpu", with_gv=True)
+    inp["xi"].zero_()
+    check_layer(w, seed_inputs=inp)
+
+
+def test_empty_shapes():
+    for T, B in ((0, 2), (3, 0)):
+        w = workloads.Workload("empty", T=T, B=B, N=64, K=4, G=1, C=4, inner=16, dtype="f32",
+                               psi="mh", reset="hard")
+        cfg = binding.config_of(w)
+        inp = to_dev(workloads.make_inputs(w, "cpu"))
+        s, _ = binding.forward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"], None)
+        g = binding.backward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"], None,
+                             inp["gs"], None)
+        torch.cuda.synchronize()
+        assert s.numel() == 0
+        for k in ("galpha", "gxi", "gzeta", "gkappa"):
+            assert torch.count_nonzero(g[k]).item() == 0
+
+
+def test_backward_is_deterministic():
+    w = scaled(WORKLOADS["token_dbg"], B=2)
+    inp = to_dev(workloads.make_inputs(w, "cpu"))
+    cfg = binding.config_of(w)
+    outs = []
+    for _ in range(2):
+        saved, scratch = binding.workspace(cfg)
+        binding.forward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"],
+                        inp["mask"], saved=saved)
+        outs.append(binding.backward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"],
+                                     inp["kappa"], inp["mask"], inp["gs"], None, saved, scratch))
+    for k in outs[0]:
+        assert torch.equal(outs[0][k], outs[1][k]), k
+
+
+def test_misaligned_device_pointer_is_rejected():
+    w = workloads.Workload("a", T=4, B=1, N=64, K=4, G=1, C=4, inner=16, dtype="f32",
+                           psi="mh", reset="hard")
+    cfg = binding.config_of(w)
+    inp = to_dev(workloads.make_inputs(w, "cpu"))
+    buf = torch.empty(inp["x"].numel() + 1, dtype=torch.float32, device="cuda")
+    x_off = buf[1:].view(inp["x"].shape)            # 4-byte offset: not 16-byte aligned
+    with pytest.raises(binding.DendSNError) as e:
+        binding.forward(cfg, x_off, inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"], None)
+    assert e.value.status == 3
+
+
+def test_autograd_function_layer_wide_alpha():
+    """DendSNFunction with the paper's scalar alpha: gradient = sum of the [C,K] one."""
+    w = workloads.Workload("ag", T=4, B=2, N=128, K=4, G=2, C=4, inner=32, dtype="f32",
+                           psi="mh", reset="hard", seed=21)
+    inp = to_dev(workloads.make_inputs(w, "cpu"))
+    cfg = binding.config_of(w)
+    x = inp["x"].clone().requires_grad_(True)
+    alpha = torch.tensor(0.7, device="cuda", requires_grad=True)
+    xi = inp["xi"].clone().requires_grad_(True)
+    zeta = inp["zeta"].clone().requires_grad_(True)
+    kappa = inp["kappa"].clone().requires_grad_(True)
+    s = binding.DendSNFunction.apply(x, alpha, xi, zeta, kappa, None, cfg)
+    (s * inp["gs"]).sum().backward()
+    full = inp["alpha"].clone().fill_(0.7)
+    ref = binding.backward(cfg, inp["x"], full, inp["xi"], inp["zeta"], inp["kappa"], None,
+                           inp["gs"], None, *binding.workspace(cfg))
+    torch.cuda.synchronize()
+    assert torch.allclose(alpha.grad, ref["galpha"].sum(), rtol=1e-5, atol=1e-6)
+    assert torch.equal(x.grad, ref["gx"])
+    assert torch.equal(kappa.grad, ref["gkappa"])
+
+
+# ------------------------------------------------------------------ full size, sampled
+def sample_neurons(w, count, seed):
+    rng = np.random.default_rng(seed)
+    flat = rng.choice(w.B * w.N, size=min(count, w.B * w.N), replace=False)
+    flat.sort()
+    return flat // w.N, flat % w.N
+
+
+@pytest.mark.parametrize("name", list(WORKLOADS))
+def test_full_size_sampled(name):
+    w = WORKLOADS[name]
+    cfg = binding.config_of(w)
+    inp = workloads.make_inputs(w, "cuda")          # full size, generated on the device
+    b_idx, n_idx = sample_neurons(w, 3000, seed=w.seed)
+    bt, nt = torch.from_numpy(b_idx).cuda(), torch.from_numpy(n_idx).cuda()
+
+    # oracle on the sampled neurons (independent of the rest of the layer)
+    xs = inp["x"][:, bt, nt, :].cpu()                                  # [T, M, K]
+    chan = ((n_idx // w.inner) % w.C).astype(np.int32)
+    mrow = (n_idx if w.mask_per_neuron else chan).astype(np.int32)
+    ocfg = oracle.OracleConfig(T=w.T, K=w.K, G=w.G, C=w.C, psi=w.psi, reset=w.reset,
+                               theta=w.theta, beta=w.beta)
+    prm = [inp[k].cpu() for k in ("alpha", "xi", "zeta", "kappa")]
+    mask = None if inp["mask"] is None else inp["mask"].cpu()
+    s_o, v_o = oracle.forward(ocfg, xs, chan, mrow, *prm, mask)
+    first = first_ambiguous_step(v_o, w.theta)
+    keep = first == w.T
+
+    # upstream gradient: zero except on the unambiguous sampled neurons
+    gs_sample = torch.zeros_like(inp["gs"])
+    kb, kn = bt[torch.from_numpy(keep).cuda()], nt[torch.from_numpy(keep).cuda()]
+    gs_sample[:, kb, kn] = inp["gs"][:, kb, kn]
+
+    saved, scratch = binding.workspace(cfg)
+    s, v = binding.forward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"],
+                           inp["mask"], want_v=True, saved=saved)
+    g = binding.backward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"],
+                         inp["mask"], gs_sample, None, saved, scratch)
+    torch.cuda.synchronize()
+    got_s = oracle.to_f64(s[:, bt, nt])
+    got_v = oracle.to_f64(v[:, bt, nt])
+    got_gx = oracle.to_f64(g["gx"][:, bt, nt, :])
+    t_idx = np.arange(w.T)[:, None]
+    assert_close("V^s", got_v, v_o, V_RTOL, 0.0, mask=t_idx <= first[None], atol_abs=V_ATOL)
+    sm = t_idx < first[None]
+    assert np.array_equal(got_s[sm], s_o[sm])
+
+    ref = oracle.backward(ocfg, xs, chan, mrow, *prm, mask, gs_sample[:, bt, nt].cpu())
+    rt, ar = (BF16_RTOL, BF16_ATOL_REL) if w.dtype == "bf16" else (G_RTOL, G_ATOL_REL)
+    assert_close("grad_x", got_gx, ref["gx"], rt, ar)
+    for k in ("galpha", "gxi", "gzeta", "gkappa"):
+        assert_close(k, oracle.to_f64(g[k]), ref[k], G_RTOL, G_ATOL_REL)
+    # every non-sampled neuron received zero upstream gradient: its grad_x is zero
+    gx_abs = g["gx"].abs().sum(dim=(0, 3))
+    gx_abs[bt, nt] = 0
+    assert torch.count_nonzero(gx_abs).item() == 0
