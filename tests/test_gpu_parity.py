@@ -85,6 +85,15 @@ def test_time_lengths_and_checkpoint_chunks(T):
     check_layer(w)
 
 
+@pytest.mark.parametrize("T", [5, 9, 13])
+def test_several_rows_per_thread_with_ragged_time(T):
+    # 640 rows of 1024 neurons: each thread walks R > 1 rows, so the prefetch of the
+    # next row crosses a ragged last chunk (T not a multiple of the load batch / chunk)
+    w = workloads.Workload("rows", T=T, B=640, N=1024, K=4, G=1, C=2, inner=512, dtype="f32",
+                           psi="mh", reset="hard", seed=30 + T)
+    check_layer(w, with_gv=False)
+
+
 def test_ragged_column_tiles_and_odd_inner():
     # P = C*inner = 300: not a multiple of any tile width; inner = 100 is not a power of 2
     w = workloads.Workload("ragged", T=5, B=3, N=600, K=4, G=1, C=3, inner=100, dtype="f32",
