@@ -44,6 +44,8 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="conv")
     ap.add_argument("--psi", choices=["mh", "identity"], default=None)
+    ap.add_argument("--batch", type=int, default=None,
+                    help="override the workload's batch B (smaller profiling captures)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU time of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -207,6 +209,8 @@ def workload_of(args):
     w = WORKLOADS[args.workload]
     if args.psi:
         w = w.with_(psi=args.psi)
+    if args.batch:
+        w = w.with_(B=args.batch)
     return w
 
 

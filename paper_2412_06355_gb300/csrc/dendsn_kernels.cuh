@@ -6,27 +6,29 @@
 // one column, hence one parameter set, for its whole life. A block is a tile of
 // TXn columns x TY row lanes; each neuron is served by LPN adjacent lanes of one
 // warp that own KT = K / LPN compartments each (16 bytes of fp32 input per step,
-// one 128-bit load). A thread walks up to R rows of its column; for each row it
-// walks the T steps in chunks. The loads of the next chunk (or next row) are
-// issued right after the current chunk's values are taken, so loads stay in
-// flight without a second register buffer.
+// one 128-bit load). A thread walks up to R rows of its column, and each row's T
+// steps in order. Loads run a fixed number of steps ahead of use through a small
+// ring of registers, across chunk and row boundaries.
 //
 // Forward (Eqs. methods-compartment .. methods-lif-fire): V^d, V^s and S stay in
 // registers across all T steps; the HBM traffic per step is the K inputs read and
 // the spike written (plus an optional V^s write and, when T > L, a checkpoint of
 // (V^d, V^s) every L steps).
 //
-// Backward (BPTT with the arctan surrogate, Eq. methods-sg): chunks are visited
-// in reverse; each is recomputed from its checkpoint (or from zero state) with the
-// forward's step function, so recomputed potentials and spikes are bit-identical
-// to the forward's; then the reverse-time recursion runs in registers and writes
-// grad_x. Parameter-gradient partials stay in registers per thread, are reduced
-// per channel inside the block in a fixed order (segmented warp shuffles, then
-// shared memory), written to scratch, and summed over blocks in a fixed order by a
+// Backward (BPTT with the arctan surrogate, Eq. methods-sg): chunks of L steps are
+// visited in reverse; each is recomputed from its checkpoint (or from zero state)
+// with the forward's step function, so recomputed potentials and spikes are
+// bit-identical to the forward's; then the reverse-time recursion runs and writes
+// grad_x. Parameter-gradient partials stay in registers per thread, are reduced per
+// channel inside the block in a fixed order (segmented warp shuffles, then shared
+// memory), written to scratch, and summed over blocks in a fixed order by a
 // finalize kernel: the parameter gradients are deterministic.
 //
-// The loop nests use 32-bit counters and pointer increments; the only 64-bit
-// divisions happen once per thread.
+// Arithmetic. With one compartment per branch (G = 1) the per-compartment work is
+// done two compartments at a time with the paired fp32 instructions of sm_100+
+// (__ffma2_rn and friends round each component exactly like __fmaf_rn), which
+// halves the floating-point instruction count; G > 1 uses a scalar engine.
+// Address arithmetic is pointer increments; 64-bit divisions happen once per thread.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -54,10 +56,13 @@ template <int KT> struct Vec<float, KT> {
         else if constexpr (KT == 2) { v[0] = r.x; v[1] = r.y; }
         else { v[0] = r; }
     }
+    static __device__ __forceinline__ Raw pack(const float (&v)[KT]) {
+        if constexpr (KT == 4) return make_float4(v[0], v[1], v[2], v[3]);
+        else if constexpr (KT == 2) return make_float2(v[0], v[1]);
+        else return v[0];
+    }
     static __device__ __forceinline__ void store(float *p, const float (&v)[KT]) {
-        if constexpr (KT == 4) __stcs(reinterpret_cast<float4 *>(p), make_float4(v[0], v[1], v[2], v[3]));
-        else if constexpr (KT == 2) __stcs(reinterpret_cast<float2 *>(p), make_float2(v[0], v[1]));
-        else __stcs(p, v[0]);
+        __stcs(reinterpret_cast<Raw *>(p), pack(v));
     }
 };
 
@@ -159,62 +164,299 @@ __device__ __forceinline__ float surrogate(float x) {
     return fast_rcp(__fmaf_rn(__fmul_rn(pi2, x), x, 1.f));
 }
 
-// ---------------------------------------------------------------- the step
-// Per-lane parameters of one neuron (KT compartments, KTb = KT/G branches).
-template <int KT, int G>
-struct LaneParams {
-    static constexpr int KTb = KT / G;
-    float a[KT];     // alpha (0 for a Stateless Dendrite)
-    float nxi[KT];   // -xi / zeta
-    float iz[KTb];   // 1 / zeta
-    float km[KTb];   // kappa * mask
-    float mk[KTb];   // mask (0/1)
-};
+__device__ __forceinline__ float2 f2(float a) { return make_float2(a, a); }
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) { return __fadd2_rn(a, b); }
+__device__ __forceinline__ float2 neg2(float2 a) { return make_float2(-a.x, -a.y); }
 
-// Affine input of compartment i: u = (V^d - xi) / zeta, evaluated as V^d/zeta - xi/zeta.
+// Per-lane parameters as loaded (KT compartments, KTb = KT/G branches).
 template <int KT, int G>
-__device__ __forceinline__ float affine(const LaneParams<KT, G> &lp, float vd, int i) {
-    return __fmaf_rn(vd, lp.iz[i / G], lp.nxi[i]);
+__device__ __forceinline__ void load_param_arrays(const Params &P, const Geometry &g, int chan,
+                                                  int sub, float (&a)[KT], float (&nxi)[KT],
+                                                  float (&iz)[KT / G], float (&km)[KT / G],
+                                                  float (&mk)[KT / G]) {
+    constexpr int KTb = KT / G;
+#pragma unroll
+    for (int b = 0; b < KTb; ++b) {
+        iz[b] = __frcp_rn(__ldg(P.zeta + (int64_t)chan * g.Kb + sub * KTb + b));
+        mk[b] = 1.f;
+    }
+#pragma unroll
+    for (int i = 0; i < KT; ++i) {
+        const int k = sub * KT + i;
+        a[i] = P.stateless ? 0.f : __ldg(P.alpha + (int64_t)chan * g.K + k);
+        nxi[i] = -__fmul_rn(__ldg(P.xi + (int64_t)chan * g.K + k), iz[i / G]);   // -xi / zeta
+    }
+    if (P.mask_mode == 1) load_mask<KTb>(P.mask + (int64_t)chan * g.Kb + sub * KTb, mk);
+#pragma unroll
+    for (int b = 0; b < KTb; ++b)
+        km[b] = __fmul_rn(__ldg(P.kappa + (int64_t)chan * g.Kb + sub * KTb + b), mk[b]);
 }
 
-// One compartment + branch step of one lane: advances V^d in place, stores the
-// branch Gaussians e^{-r^2/2} (Mexican hat only) in eb, and returns the lane's share
-// of Z[t] (Eqs. methods-compartment, -branch-aggregation, -mexican-hat,
-// -soma-input, -residual). Explicit rounding intrinsics keep the forward kernel and
-// the backward's recompute bit-identical.
+// kappa * m and m for the neuron n of a per-neuron mask (mask_mode 2).
+template <int KTb>
+__device__ __forceinline__ void load_neuron_mask(const Params &P, const Geometry &g, int64_t n,
+                                                 int chan, int sub, float (&km)[KTb],
+                                                 float (&mk)[KTb]) {
+    load_mask<KTb>(P.mask + n * g.Kb + sub * KTb, mk);
+#pragma unroll
+    for (int b = 0; b < KTb; ++b)
+        km[b] = __fmul_rn(__ldg(P.kappa + (int64_t)chan * g.Kb + sub * KTb + b), mk[b]);
+}
+
+// ================================================================ paired engine, G = 1
+// Compartment i is branch i. u = V^d/zeta - xi/zeta; r = |u|.
+template <int KT, int PSI>
+struct PairArith {
+    static constexpr int N2 = KT / 2;
+    static constexpr int KTb = KT;
+    struct LP { float2 a[N2], nxi[N2], iz[N2], km[N2], mk[N2]; };
+    struct St { float2 v[N2]; };
+    struct Acc { float2 ga[N2], ngxi[N2], ngz[N2], gk[N2]; };   // ngxi, ngz: negated sums
+
+    static __device__ __forceinline__ void load(const Params &P, const Geometry &g, int chan, int sub, LP &lp) {
+        float a[KT], nxi[KT], iz[KT], km[KT], mk[KT];
+        load_param_arrays<KT, 1>(P, g, chan, sub, a, nxi, iz, km, mk);
+#pragma unroll
+        for (int m = 0; m < N2; ++m) {
+            lp.a[m] = make_float2(a[2 * m], a[2 * m + 1]);
+            lp.nxi[m] = make_float2(nxi[2 * m], nxi[2 * m + 1]);
+            lp.iz[m] = make_float2(iz[2 * m], iz[2 * m + 1]);
+            lp.km[m] = make_float2(km[2 * m], km[2 * m + 1]);
+            lp.mk[m] = make_float2(mk[2 * m], mk[2 * m + 1]);
+        }
+    }
+    static __device__ __forceinline__ void neuron_mask(const Params &P, const Geometry &g, int64_t n, int chan, int sub, LP &lp) {
+        float km[KT], mk[KT];
+        load_neuron_mask<KT>(P, g, n, chan, sub, km, mk);
+#pragma unroll
+        for (int m = 0; m < N2; ++m) {
+            lp.km[m] = make_float2(km[2 * m], km[2 * m + 1]);
+            lp.mk[m] = make_float2(mk[2 * m], mk[2 * m + 1]);
+        }
+    }
+    static __device__ __forceinline__ void zero(St &s) {
+#pragma unroll
+        for (int m = 0; m < N2; ++m) s.v[m] = f2(0.f);
+    }
+    static __device__ __forceinline__ void to_array(const St &s, float (&v)[KT]) {
+#pragma unroll
+        for (int m = 0; m < N2; ++m) { v[2 * m] = s.v[m].x; v[2 * m + 1] = s.v[m].y; }
+    }
+    static __device__ __forceinline__ void from_array(St &s, const float (&v)[KT]) {
+#pragma unroll
+        for (int m = 0; m < N2; ++m) s.v[m] = make_float2(v[2 * m], v[2 * m + 1]);
+    }
+    // Eqs. methods-compartment, -branch-aggregation, -mexican-hat, -soma-input.
+    static __device__ __forceinline__ float step(const LP &lp, St &vd, const float (&x)[KT]) {
+        float2 zp = f2(0.f);
+#pragma unroll
+        for (int m = 0; m < N2; ++m) {
+            vd.v[m] = ffma2(lp.a[m], vd.v[m], make_float2(x[2 * m], x[2 * m + 1]));
+            const float2 u = ffma2(vd.v[m], lp.iz[m], lp.nxi[m]);
+            float2 y;
+            if constexpr (PSI == PSI_MEXHAT) {
+                const float2 ss = fmul2(u, u);
+                const float2 t = fmul2(f2(kNegHalfLog2e), ss);
+                const float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
+                y = ffma2(neg2(ss), e, e);                       // (1 - r^2) e^{-r^2/2}
+            } else {
+                y = make_float2(fabsf(u.x), fabsf(u.y));         // r
+            }
+            zp = (m == 0) ? fmul2(lp.km[m], y) : ffma2(lp.km[m], y, zp);
+        }
+        return __fadd_rn(zp.x, zp.y);
+    }
+    static __device__ __forceinline__ void acc_zero(Acc &c) {
+#pragma unroll
+        for (int m = 0; m < N2; ++m) { c.ga[m] = f2(0.f); c.ngxi[m] = f2(0.f); c.ngz[m] = f2(0.f); c.gk[m] = f2(0.f); }
+    }
+    // [alpha KT | xi KT | zeta KTb | kappa KTb]
+    static __device__ __forceinline__ void acc_export(const Acc &c, float *v) {
+#pragma unroll
+        for (int m = 0; m < N2; ++m) {
+            v[2 * m] = c.ga[m].x;                v[2 * m + 1] = c.ga[m].y;
+            v[KT + 2 * m] = -c.ngxi[m].x;        v[KT + 2 * m + 1] = -c.ngxi[m].y;
+            v[2 * KT + 2 * m] = -c.ngz[m].x;     v[2 * KT + 2 * m + 1] = -c.ngz[m].y;
+            v[3 * KT + 2 * m] = c.gk[m].x;       v[3 * KT + 2 * m + 1] = c.gk[m].y;
+        }
+    }
+    // One reverse step: V^d[t] (vdt), V^d[t-1] (vdp) and dL/dZ[t] (dz) update the
+    // dendritic adjoint Ad = dL/dV^d (reverse scan of Eq. methods-compartment), the
+    // parameter-gradient partials, and give dL/dX[t] = Ad (+ res).
+    static __device__ __forceinline__ void backward(const LP &lp, const St &vdt, const St &vdp, float dz,
+                                                    St &Ad, Acc &acc, float res, float (&gx)[KT]) {
+        const float2 dz2 = f2(dz);
+#pragma unroll
+        for (int m = 0; m < N2; ++m) {
+            const float2 u = ffma2(vdt.v[m], lp.iz[m], lp.nxi[m]);
+            const float2 gy = fmul2(lp.km[m], dz2);              // dL/dY
+            float2 y, d, grr;                                    // Y, dL/dV^d direct, (dL/dr) r
+            if constexpr (PSI == PSI_MEXHAT) {
+                const float2 ss = fmul2(u, u);
+                const float2 t = fmul2(f2(kNegHalfLog2e), ss);
+                const float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
+                y = ffma2(neg2(ss), e, e);
+                // psi'(r) / r = (r^2 - 3) e^{-r^2/2}: du = q u
+                const float2 q = fmul2(fmul2(fadd2(ss, f2(-3.f)), e), gy);
+                d = fmul2(fmul2(q, u), lp.iz[m]);
+                grr = fmul2(ss, q);
+            } else {
+                const float2 r = make_float2(fabsf(u.x), fabsf(u.y));
+                const float2 gu = make_float2(u.x > 0.f ? gy.x : (u.x < 0.f ? -gy.x : 0.f),
+                                              u.y > 0.f ? gy.y : (u.y < 0.f ? -gy.y : 0.f));
+                y = r;
+                d = fmul2(gu, lp.iz[m]);
+                grr = fmul2(gy, r);
+            }
+            acc.ngxi[m] = fadd2(acc.ngxi[m], d);                 // dxi = -direct
+            acc.ngz[m] = ffma2(grr, lp.iz[m], acc.ngz[m]);       // dzeta = -(dL/dr) r / zeta
+            acc.gk[m] = ffma2(fmul2(lp.mk[m], y), dz2, acc.gk[m]);
+            Ad.v[m] = ffma2(lp.a[m], Ad.v[m], d);
+            acc.ga[m] = ffma2(Ad.v[m], vdp.v[m], acc.ga[m]);
+            gx[2 * m] = __fadd_rn(Ad.v[m].x, res);
+            gx[2 * m + 1] = __fadd_rn(Ad.v[m].y, res);
+        }
+    }
+};
+
+// ================================================================ scalar engine, any G
 template <int KT, int G, int PSI>
-__device__ __forceinline__ float dendrite_step(const LaneParams<KT, G> &lp, float (&vd)[KT],
-                                               const float (&x)[KT], bool residual, float inv_k,
-                                               float (&eb)[KT / G]) {
-#pragma unroll
-    for (int i = 0; i < KT; ++i) vd[i] = __fmaf_rn(lp.a[i], vd[i], x[i]);
-    float zp = 0.f;
-#pragma unroll
-    for (int b = 0; b < KT / G; ++b) {
-        float ss = 0.f, u0 = 0.f;
-#pragma unroll
-        for (int g = 0; g < G; ++g) {
-            const float u = affine(lp, vd[b * G + g], b * G + g);
-            if (g == 0) u0 = u;
-            ss = (g == 0) ? __fmul_rn(u, u) : __fmaf_rn(u, u, ss);
-        }
-        float y;
-        if constexpr (PSI == PSI_MEXHAT) {
-            const float e = gauss_half(ss);
-            eb[b] = e;
-            y = __fmaf_rn(-ss, e, e);                     // (1 - r^2) e^{-r^2/2}
-        } else {
-            y = (G == 1) ? fabsf(u0) : sqrtf(ss);         // r
-        }
-        zp = __fmaf_rn(lp.km[b], y, zp);
+struct ScalarArith {
+    static constexpr int KTb = KT / G;
+    struct LP { float a[KT], nxi[KT], iz[KTb], km[KTb], mk[KTb]; };
+    struct St { float v[KT]; };
+    struct Acc { float ga[KT], gxi[KT], gz[KTb], gk[KTb]; };
+
+    static __device__ __forceinline__ void load(const Params &P, const Geometry &g, int chan, int sub, LP &lp) {
+        load_param_arrays<KT, G>(P, g, chan, sub, lp.a, lp.nxi, lp.iz, lp.km, lp.mk);
     }
-    if (residual) {
-        float xs = 0.f;
-#pragma unroll
-        for (int i = 0; i < KT; ++i) xs = __fadd_rn(xs, x[i]);
-        zp = __fmaf_rn(xs, inv_k, zp);
+    static __device__ __forceinline__ void neuron_mask(const Params &P, const Geometry &g, int64_t n, int chan, int sub, LP &lp) {
+        load_neuron_mask<KTb>(P, g, n, chan, sub, lp.km, lp.mk);
     }
-    return zp;
+    static __device__ __forceinline__ void zero(St &s) {
+#pragma unroll
+        for (int i = 0; i < KT; ++i) s.v[i] = 0.f;
+    }
+    static __device__ __forceinline__ void to_array(const St &s, float (&v)[KT]) {
+#pragma unroll
+        for (int i = 0; i < KT; ++i) v[i] = s.v[i];
+    }
+    static __device__ __forceinline__ void from_array(St &s, const float (&v)[KT]) {
+#pragma unroll
+        for (int i = 0; i < KT; ++i) s.v[i] = v[i];
+    }
+    static __device__ __forceinline__ float affine(const LP &lp, float vd, int i) {
+        return __fmaf_rn(vd, lp.iz[i / G], lp.nxi[i]);
+    }
+    // Eqs. methods-compartment, -branch-aggregation, -mexican-hat, -soma-input.
+    static __device__ __forceinline__ float step(const LP &lp, St &vd, const float (&x)[KT]) {
+#pragma unroll
+        for (int i = 0; i < KT; ++i) vd.v[i] = __fmaf_rn(lp.a[i], vd.v[i], x[i]);
+        float zp = 0.f;
+#pragma unroll
+        for (int b = 0; b < KTb; ++b) {
+            float ss = 0.f, u0 = 0.f;
+#pragma unroll
+            for (int q = 0; q < G; ++q) {
+                const float u = affine(lp, vd.v[b * G + q], b * G + q);
+                if (q == 0) u0 = u;
+                ss = (q == 0) ? __fmul_rn(u, u) : __fmaf_rn(u, u, ss);
+            }
+            float y;
+            if constexpr (PSI == PSI_MEXHAT) {
+                const float e = gauss_half(ss);
+                y = __fmaf_rn(-ss, e, e);                     // (1 - r^2) e^{-r^2/2}
+            } else {
+                y = (G == 1) ? fabsf(u0) : sqrtf(ss);         // r
+            }
+            zp = __fmaf_rn(lp.km[b], y, zp);
+        }
+        return zp;
+    }
+    static __device__ __forceinline__ void acc_zero(Acc &c) {
+#pragma unroll
+        for (int i = 0; i < KT; ++i) { c.ga[i] = 0.f; c.gxi[i] = 0.f; }
+#pragma unroll
+        for (int b = 0; b < KTb; ++b) { c.gz[b] = 0.f; c.gk[b] = 0.f; }
+    }
+    static __device__ __forceinline__ void acc_export(const Acc &c, float *v) {
+#pragma unroll
+        for (int i = 0; i < KT; ++i) { v[i] = c.ga[i]; v[KT + i] = c.gxi[i]; }
+#pragma unroll
+        for (int b = 0; b < KTb; ++b) { v[2 * KT + b] = c.gz[b]; v[2 * KT + KTb + b] = c.gk[b]; }
+    }
+    static __device__ __forceinline__ void backward(const LP &lp, const St &vdt, const St &vdp, float dz,
+                                                    St &Ad, Acc &acc, float res, float (&gx)[KT]) {
+        float direct[KT];
+#pragma unroll
+        for (int b = 0; b < KTb; ++b) {
+            float u[G];
+            float ss = 0.f;
+#pragma unroll
+            for (int q = 0; q < G; ++q) {
+                u[q] = affine(lp, vdt.v[b * G + q], b * G + q);
+                ss = (q == 0) ? __fmul_rn(u[q], u[q]) : __fmaf_rn(u[q], u[q], ss);
+            }
+            const float gy = __fmul_rn(lp.km[b], dz);       // dL/dY_b
+            float y, grr;                                    // Y_b and (dL/dr_b) * r_b
+            if constexpr (PSI == PSI_MEXHAT) {
+                const float e = gauss_half(ss);
+                y = __fmaf_rn(-ss, e, e);
+                // psi'(r) / r = (r^2 - 3) e^{-r^2/2}, so du_i = q u_i with no division
+                const float qq = __fmul_rn(__fmul_rn(__fsub_rn(ss, 3.f), e), gy);
+#pragma unroll
+                for (int q = 0; q < G; ++q) {
+                    const float d = __fmul_rn(__fmul_rn(qq, u[q]), lp.iz[b]);
+                    direct[b * G + q] = d;
+                    acc.gxi[b * G + q] = __fsub_rn(acc.gxi[b * G + q], d);
+                }
+                grr = __fmul_rn(ss, qq);
+            } else {
+                float r;
+                if constexpr (G == 1) {
+                    r = fabsf(u[0]);
+                    const float gu = (u[0] > 0.f) ? gy : ((u[0] < 0.f) ? -gy : 0.f);
+                    const float d = __fmul_rn(gu, lp.iz[b]);
+                    direct[b] = d;
+                    acc.gxi[b] = __fsub_rn(acc.gxi[b], d);
+                } else {
+                    r = sqrtf(ss);
+                    const float qq = (r > 0.f) ? __fdiv_rn(gy, r) : 0.f;   // subgradient 0 at r = 0
+#pragma unroll
+                    for (int q = 0; q < G; ++q) {
+                        const float d = __fmul_rn(__fmul_rn(qq, u[q]), lp.iz[b]);
+                        direct[b * G + q] = d;
+                        acc.gxi[b * G + q] = __fsub_rn(acc.gxi[b * G + q], d);
+                    }
+                }
+                y = r;
+                grr = __fmul_rn(gy, r);
+            }
+            acc.gz[b] = __fmaf_rn(-grr, lp.iz[b], acc.gz[b]);
+            acc.gk[b] = __fmaf_rn(__fmul_rn(lp.mk[b], y), dz, acc.gk[b]);
+        }
+#pragma unroll
+        for (int i = 0; i < KT; ++i) {
+            Ad.v[i] = __fmaf_rn(lp.a[i], Ad.v[i], direct[i]);
+            gx[i] = __fadd_rn(Ad.v[i], res);
+            acc.ga[i] = __fmaf_rn(Ad.v[i], vdp.v[i], acc.ga[i]);
+        }
+    }
+};
+
+template <int KT, int G, int PSI>
+using Arith = typename std::conditional<(G == 1 && KT % 2 == 0), PairArith<KT, PSI>,
+                                        ScalarArith<KT, G, PSI>>::type;
+
+// Eq. methods-residual: the lane's share of sum_i X_i (same order in forward and recompute).
+template <int KT>
+__device__ __forceinline__ float lane_input_sum(const float (&x)[KT]) {
+    float xs = x[0];
+#pragma unroll
+    for (int i = 1; i < KT; ++i) xs = __fadd_rn(xs, x[i]);
+    return xs;
 }
 
 // Sum of the LPN lanes' shares (xor butterfly: every lane gets the same bits).
@@ -224,6 +466,15 @@ __device__ __forceinline__ float lanes_sum(float v) {
     if constexpr (LPN >= 4) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, 2));
     if constexpr (LPN >= 8) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, 4));
     return v;
+}
+
+// Z[t] of the neuron: the lane's branch share (plus its residual share), summed over lanes.
+template <typename AR, int KT, int LPN>
+__device__ __forceinline__ float soma_input(const typename AR::LP &lp, typename AR::St &vd,
+                                            const float (&x)[KT], bool residual, float inv_k) {
+    float zp = AR::step(lp, vd, x);
+    if (residual) zp = __fmaf_rn(lane_input_sum<KT>(x), inv_k, zp);
+    return lanes_sum<LPN>(zp);
 }
 
 // LIF soma charge with the reset folded in: hard V = beta (1 - S) V + Z
@@ -265,182 +516,99 @@ __device__ __forceinline__ ThreadPos thread_pos(const Geometry &g) {
     return t;
 }
 
-template <int KT, int G>
-__device__ __forceinline__ void load_lane_params(const Params &P, const Geometry &g, int chan,
-                                                 int sub, LaneParams<KT, G> &lp) {
-    constexpr int KTb = KT / G;
-#pragma unroll
-    for (int b = 0; b < KTb; ++b) {
-        lp.iz[b] = __frcp_rn(__ldg(P.zeta + (int64_t)chan * g.Kb + sub * KTb + b));
-        lp.mk[b] = 1.f;
-    }
-#pragma unroll
-    for (int i = 0; i < KT; ++i) {
-        const int k = sub * KT + i;
-        lp.a[i] = P.stateless ? 0.f : __ldg(P.alpha + (int64_t)chan * g.K + k);
-        lp.nxi[i] = -__fmul_rn(__ldg(P.xi + (int64_t)chan * g.K + k), lp.iz[i / G]);
-    }
-    if (P.mask_mode == 1) load_mask<KTb>(P.mask + (int64_t)chan * g.Kb + sub * KTb, lp.mk);
-#pragma unroll
-    for (int b = 0; b < KTb; ++b)
-        lp.km[b] = __fmul_rn(__ldg(P.kappa + (int64_t)chan * g.Kb + sub * KTb + b), lp.mk[b]);
-}
-
-// Per-neuron mask (mask_mode 2): kappa * m for the neuron in column p of row o.
-template <int KT, int G>
-__device__ __forceinline__ void apply_neuron_mask(const Params &P, const Geometry &g,
-                                                  int64_t o, int p, int chan, int sub,
-                                                  LaneParams<KT, G> &lp) {
-    constexpr int KTb = KT / G;
-    const int64_t n = (o * g.P + p) % g.N;
-    load_mask<KTb>(P.mask + n * g.Kb + sub * KTb, lp.mk);
-#pragma unroll
-    for (int b = 0; b < KTb; ++b)
-        lp.km[b] = __fmul_rn(__ldg(P.kappa + (int64_t)chan * g.Kb + sub * KTb + b), lp.mk[b]);
-}
-
 // ---------------------------------------------------------------- forward
-// One load batch = kFwdBatch steps; checkpoints every g.L steps (g.L is a power of
-// two and a multiple of the batch, so they fall on batch ends).
+// x is prefetched kFwdBatch steps ahead of use (a ring of kFwdBatch registers);
+// checkpoints every g.L steps (g.L is a power of two and a multiple of the batch).
 template <int K, int G, int PSI, typename XT>
-__global__ void __launch_bounds__(kThreads, 3)
+__global__ void __launch_bounds__(kThreads, 2)
 dendsn_forward_kernel(const FwdArgs A) {
     constexpr int KT = (K < 4) ? K : 4;
     constexpr int LPN = K / KT;
-    constexpr int KTb = KT / G;
     constexpr int L = kFwdBatch;
     using V = Vec<XT, KT>;
+    using AR = Arith<KT, G, PSI>;
     const Geometry &g = A.g;
     const Params &P = A.p;
     const ThreadPos pos = thread_pos<LPN>(g);
     if (pos.nrows == 0) return;                  // whole warps: rows are uniform per warp
-    LaneParams<KT, G> lp;
-    load_lane_params<KT, G>(P, g, pos.chan, pos.sub, lp);
+    typename AR::LP lp;
+    AR::load(P, g, pos.chan, pos.sub, lp);
     const float inv_k = 1.f / (float)K;
     const int T = g.T;
-    const int nb = (T + L - 1) / L;              // load batches per row
-    const int64_t stepX = g.BN * K;              // elements between steps of x
+    const int nb = (T + L - 1) / L;              // batches per row
+    const int64_t sX = g.BN * K;                 // x elements between steps
+    const int64_t BN = g.BN;
     const int64_t j0 = pos.row0 * g.P + pos.p;   // first neuron of this thread
     const int64_t jstep = (int64_t)pos.rstride * g.P;
-    const XT *__restrict__ x0 = static_cast<const XT *>(A.x) + j0 * K + pos.sub * KT;
-    XT *__restrict__ s0 = static_cast<XT *>(A.spikes) + j0;
-    const bool write_ck = (A.ck_vd != nullptr) && g.n_ck > 0;
+    const int64_t rX = jstep * K;                // x elements between this thread's rows
+    const XT *__restrict__ xrow = static_cast<const XT *>(A.x) + j0 * K + pos.sub * KT;
+    XT *__restrict__ srow = static_cast<XT *>(A.spikes) + j0;
+    float *vrow = A.v_out ? A.v_out + j0 : nullptr;
+    const bool write_ck = (A.ck_vd != nullptr) && g.n_ck > 0 && pos.active;
     const bool store = pos.active && pos.sub == 0;
+    const bool residual = P.residual != 0;
 
     typename V::Raw xb[L];
+    {
+        const XT *p = xrow;
 #pragma unroll
-    for (int tt = 0; tt < L; ++tt)
-        if (tt < T) xb[tt] = V::load(x0 + tt * stepX);
-
+        for (int tt = 0; tt < L; ++tt) {
+            if (tt < T) xb[tt] = V::load(p);
+            p += sX;
+        }
+    }
+    int64_t j = j0;
     for (int i = 0; i < pos.nrows; ++i) {
-        const XT *xr = x0 + i * jstep * K;
-        const int64_t j = j0 + i * jstep;
-        if (P.mask_mode == 2)
-            apply_neuron_mask<KT, G>(P, g, pos.row0 + (int64_t)i * pos.rstride, pos.p, pos.chan,
-                                     pos.sub, lp);
-        float vd[KT];
-#pragma unroll
-        for (int k = 0; k < KT; ++k) vd[k] = 0.f;
+        if (P.mask_mode == 2) AR::neuron_mask(P, g, j % g.N, pos.chan, pos.sub, lp);
+        typename AR::St vd;
+        AR::zero(vd);
         float v = 0.f;
         bool s = false;
+        XT *sp = srow;
+        float *vp = vrow;
         for (int c = 0; c < nb; ++c) {
             const int t0 = c * L;
+            const int ncur = min(L, T - t0);                       // steps of this batch
             const bool same_row = c + 1 < nb;
             const bool has_next = same_row || (i + 1 < pos.nrows);
-            const int tn = same_row ? t0 + L : 0;
-            const XT *xn = same_row ? xr + tn * stepX : xr + jstep * K;
+            // next batch: later in this row, or the start of the next row
+            const XT *xn = same_row ? xrow + (int64_t)(t0 + L) * sX : xrow + rX;
+            const int nnext = !has_next ? 0 : (same_row ? min(L, T - t0 - L) : min(L, T));
 #pragma unroll
             for (int tt = 0; tt < L; ++tt) {
                 float xv[KT];
                 V::unpack(xb[tt], xv);
-                // refill slot tt for the next unit right after its value is taken
-                if (has_next && tn + tt < T) xb[tt] = V::load(xn + tt * stepX);
-                const int t = t0 + tt;
-                if (t < T) {
-                    float eb[KTb];
-                    const float z = lanes_sum<LPN>(
-                        dendrite_step<KT, G, PSI>(lp, vd, xv, P.residual != 0, inv_k, eb));
+                // refill slot tt right after its value is taken
+                if (tt < nnext) xb[tt] = V::load(xn);
+                xn += sX;
+                if (tt < ncur) {
+                    const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
                     v = soma_charge(z, v, s, P);
                     s = v >= P.theta;                      // Eq. methods-lif-fire
                     if (store) {
-                        Scalar<XT>::store_spike(s0 + t * g.BN + i * jstep, s);
-                        if (A.v_out) __stcs(A.v_out + t * g.BN + j, v);
+                        Scalar<XT>::store_spike(sp, s);
+                        if (vp) __stcs(vp, v);
                     }
+                    sp += BN;
+                    if (vp) vp += BN;
                 }
             }
-            if (write_ck && t0 + L < T && ((t0 + L) & (g.L - 1)) == 0 && pos.active) {
+            if (write_ck && t0 + L < T && ((t0 + L) & (g.L - 1)) == 0) {
                 const int ck = (t0 + L) / g.L - 1;
-                Vec<float, KT>::store(A.ck_vd + ((int64_t)ck * g.BN + j) * K + pos.sub * KT, vd);
-                if (pos.sub == 0) __stcs(A.ck_vs + (int64_t)ck * g.BN + j, v);
+                float vda[KT];
+                AR::to_array(vd, vda);
+                Vec<float, KT>::store(A.ck_vd + ((int64_t)ck * BN + j) * K + pos.sub * KT, vda);
+                if (pos.sub == 0) __stcs(A.ck_vs + (int64_t)ck * BN + j, v);
             }
         }
+        xrow += rX;
+        srow += jstep;
+        if (vrow) vrow += jstep;
+        j += jstep;
     }
 }
 
 // ---------------------------------------------------------------- backward
-template <int KT, int G>
-struct GradAcc {
-    static constexpr int KTb = KT / G;
-    float ga[KT], gxi[KT], gz[KTb], gk[KTb];
-};
-
-// Gradients through the branches of one lane at one step, from V^d[t] (vd), the
-// branch Gaussians of the recompute (eb, Mexican hat) and dL/dZ[t] (dz).
-// direct[i] = dL/dV^d_i[t] through this step's branch only.
-template <int KT, int G, int PSI>
-__device__ __forceinline__ void branch_backward(const LaneParams<KT, G> &lp,
-                                                const float (&vd)[KT], const float (&eb)[KT / G],
-                                                float dz, float (&direct)[KT],
-                                                GradAcc<KT, G> &acc) {
-#pragma unroll
-    for (int b = 0; b < KT / G; ++b) {
-        float u[G];
-        float ss = 0.f;
-#pragma unroll
-        for (int g = 0; g < G; ++g) {
-            u[g] = affine(lp, vd[b * G + g], b * G + g);
-            ss = (g == 0) ? __fmul_rn(u[g], u[g]) : __fmaf_rn(u[g], u[g], ss);
-        }
-        const float gy = __fmul_rn(lp.km[b], dz);       // dL/dY_b
-        float y, grr;                                    // Y_b and (dL/dr_b) * r_b
-        if constexpr (PSI == PSI_MEXHAT) {
-            const float e = eb[b];
-            y = __fmaf_rn(-ss, e, e);
-            // psi'(r) / r = (r^2 - 3) e^{-r^2/2}, so du_i = q u_i with no division
-            const float q = __fmul_rn(__fmul_rn(__fsub_rn(ss, 3.f), e), gy);
-#pragma unroll
-            for (int g = 0; g < G; ++g) {
-                const float d = __fmul_rn(__fmul_rn(q, u[g]), lp.iz[b]);
-                direct[b * G + g] = d;
-                acc.gxi[b * G + g] = __fsub_rn(acc.gxi[b * G + g], d);
-            }
-            grr = __fmul_rn(ss, q);
-        } else {
-            float r;
-            if constexpr (G == 1) {
-                r = fabsf(u[0]);
-                const float gu = (u[0] > 0.f) ? gy : ((u[0] < 0.f) ? -gy : 0.f);
-                const float d = __fmul_rn(gu, lp.iz[b]);
-                direct[b] = d;
-                acc.gxi[b] = __fsub_rn(acc.gxi[b], d);
-            } else {
-                r = sqrtf(ss);
-                const float q = (r > 0.f) ? __fdiv_rn(gy, r) : 0.f;   // subgradient 0 at r = 0
-#pragma unroll
-                for (int g = 0; g < G; ++g) {
-                    const float d = __fmul_rn(__fmul_rn(q, u[g]), lp.iz[b]);
-                    direct[b * G + g] = d;
-                    acc.gxi[b * G + g] = __fsub_rn(acc.gxi[b * G + g], d);
-                }
-            }
-            y = r;
-            grr = __fmul_rn(gy, r);
-        }
-        acc.gz[b] = __fmaf_rn(-grr, lp.iz[b], acc.gz[b]);
-        acc.gk[b] = __fmaf_rn(__fmul_rn(lp.mk[b], y), dz, acc.gk[b]);
-    }
-}
-
 template <int KT, int G>
 constexpr int acc_count() { return 2 * KT + 2 * (KT / G); }
 
@@ -453,193 +621,211 @@ dendsn_backward_kernel(const BwdArgs A) {
     constexpr int NA = acc_count<KT, G>();
     // L == 4 is only used for T <= 4: one chunk per row and never a checkpoint
     constexpr bool MULTI = L > 4;
-    // keep the recompute's Gaussians for the reverse pass (costs L * KTb registers)
-    constexpr bool KEEP_E = false;
+    constexpr int H = 4;                         // prefetch distance of x in steps
     using V = Vec<XT, KT>;
     using S1 = Scalar<XT>;
+    using AR = Arith<KT, G, PSI>;
+    using HistRaw = typename Vec<float, KT>::Raw;
     const Geometry &g = A.g;
     const Params &P = A.p;
     const ThreadPos pos = thread_pos<LPN>(g);
-    LaneParams<KT, G> lp;
-    load_lane_params<KT, G>(P, g, pos.chan, pos.sub, lp);
+    typename AR::LP lp;
+    AR::load(P, g, pos.chan, pos.sub, lp);
     const float inv_k = 1.f / (float)K;
     const int T = g.T;
     const int nc = MULTI ? (T + L - 1) / L : 1;  // chunks per row
-    const int64_t stepX = g.BN * K;
+    const int64_t sX = g.BN * K;
     const int64_t BN = g.BN;
     const int64_t j0 = pos.row0 * g.P + pos.p;
     const int64_t jstep = (int64_t)pos.rstride * g.P;
-    const XT *__restrict__ x0 = static_cast<const XT *>(A.x) + j0 * K + pos.sub * KT;
-    const XT *__restrict__ gs0 = static_cast<const XT *>(A.gs) + j0;
-    XT *__restrict__ gx0 = static_cast<XT *>(A.gx) + j0 * K + pos.sub * KT;
+    const int64_t rX = jstep * K;
+    const XT *__restrict__ xrow = static_cast<const XT *>(A.x) + j0 * K + pos.sub * KT;
+    const XT *__restrict__ gsrow = static_cast<const XT *>(A.gs) + j0;
+    XT *__restrict__ gxrow = static_cast<XT *>(A.gx) + j0 * K + pos.sub * KT;
+    const float *gvrow = A.gv ? A.gv + j0 : nullptr;
     const float hard_dvds = -P.beta;             // dV[t+1]/dS[t] = -beta V[t]
     const float soft_dvds = -P.beta * P.theta;   // dV[t+1]/dS[t] = -beta theta
+    const bool residual = P.residual != 0;
 
-    GradAcc<KT, G> acc;
-#pragma unroll
-    for (int i = 0; i < KT; ++i) { acc.ga[i] = 0.f; acc.gxi[i] = 0.f; }
-#pragma unroll
-    for (int b = 0; b < KTb; ++b) { acc.gz[b] = 0.f; acc.gk[b] = 0.f; }
+    extern __shared__ float4 smem_f4[];
+    HistRaw *hist = reinterpret_cast<HistRaw *>(smem_f4);                             // [L][kThreads]
+    float *hist_vs = reinterpret_cast<float *>(hist + (MULTI ? L * kThreads : 0));   // [L][kThreads]
 
-    typename V::Raw xb[L];            // inputs of the current unit, refilled with the next unit's
-    typename S1::Raw gsb[L];          // grad_spikes of the current unit
-    float ckd[KT];                    // checkpoint V^d entering the current unit
-    float ckv = 0.f;                  // checkpoint V^s entering the current unit
+    typename AR::Acc acc;
+    AR::acc_zero(acc);
+
+    typename V::Raw xb[H];            // x of the next H steps to recompute
+    typename S1::Raw gsb[L];          // grad_spikes of the current chunk
+    float ckd[KT];                    // checkpoint V^d entering the current chunk
+    float ckv = 0.f;                  // checkpoint V^s entering the current chunk
 #pragma unroll
     for (int i = 0; i < KT; ++i) ckd[i] = 0.f;
     if (pos.nrows > 0) {
-        const int c = nc - 1;
-        const int t0 = c * L;
+        const int t0 = (nc - 1) * L;
+        const XT *p = xrow + (int64_t)t0 * sX;
+        const XT *q = gsrow + (int64_t)t0 * BN;
 #pragma unroll
-        for (int tt = 0; tt < L; ++tt)
+        for (int tt = 0; tt < L; ++tt) {
             if (t0 + tt < T) {
-                xb[tt] = V::load(x0 + (t0 + tt) * stepX);
-                gsb[tt] = S1::load(gs0 + (t0 + tt) * BN);
+                if (tt < H) xb[tt < H ? tt : 0] = V::load(p);
+                gsb[tt] = S1::load(q);
             }
-        if (MULTI && c > 0) {
+            p += sX;
+            q += BN;
+        }
+        if (MULTI && nc > 1) {
             Vec<float, KT>::unpack(Vec<float, KT>::load(
-                A.ck_vd + ((int64_t)(c - 1) * BN + j0) * K + pos.sub * KT), ckd);
-            ckv = __ldcs(A.ck_vs + (int64_t)(c - 1) * BN + j0);
+                A.ck_vd + ((int64_t)(nc - 2) * BN + j0) * K + pos.sub * KT), ckd);
+            ckv = __ldcs(A.ck_vs + (int64_t)(nc - 2) * BN + j0);
         }
     }
 
+    int64_t j = j0;
     for (int i = 0; i < pos.nrows; ++i) {
-        const int64_t j = j0 + i * jstep;
-        const XT *xr = x0 + i * jstep * K;
-        const XT *gsr = gs0 + i * jstep;
-        XT *gxr = gx0 + i * jstep * K;
-        if (P.mask_mode == 2)
-            apply_neuron_mask<KT, G>(P, g, pos.row0 + (int64_t)i * pos.rstride, pos.p, pos.chan,
-                                     pos.sub, lp);
-        float Ad[KT];        // dL/dV^d[t+1], carried backwards
-#pragma unroll
-        for (int k = 0; k < KT; ++k) Ad[k] = 0.f;
-        float dvn = 0.f;     // dL/dV^s[t+1]
+        if (P.mask_mode == 2) AR::neuron_mask(P, g, j % g.N, pos.chan, pos.sub, lp);
+        typename AR::St Ad;           // dL/dV^d[t+1], carried backwards
+        AR::zero(Ad);
+        float dvn = 0.f;              // dL/dV^s[t+1]
         for (int c = nc - 1; c >= 0; --c) {
             const int t0 = c * L;
+            const int ncur = min(L, T - t0);
             // state entering the chunk: zero at t = 0, else the forward's checkpoint
-            float vd0[KT];
-#pragma unroll
-            for (int k = 0; k < KT; ++k) vd0[k] = (!MULTI || c == 0) ? 0.f : ckd[k];
+            typename AR::St vd0;
+            if (!MULTI || c == 0) {
+                AR::zero(vd0);
+            } else {
+                AR::from_array(vd0, ckd);
+            }
             const float v0 = (!MULTI || c == 0) ? 0.f : ckv;
-            // next unit: the previous chunk of this row, or the last chunk of the next row
+            // next chunk: the previous chunk of this row, or the last chunk of the next row
             const bool same_row = MULTI && c > 0;
             const bool has_next = same_row || (i + 1 < pos.nrows);
             const int cn = same_row ? c - 1 : nc - 1;
             const int tn = cn * L;
+            const int nnext = has_next ? min(L, T - tn) : 0;
             const int64_t jn = same_row ? j : j + jstep;
-            const XT *xn = (same_row ? xr : xr + jstep * K) + tn * stepX;
-            const XT *gsn = (same_row ? gsr : gsr + jstep) + tn * BN;
+            const XT *xn = (same_row ? xrow : xrow + rX) + (int64_t)tn * sX;
+            const XT *gsn = (same_row ? gsrow : gsrow + jstep) + (int64_t)tn * BN;
             if (MULTI && has_next && cn > 0) {
                 Vec<float, KT>::unpack(Vec<float, KT>::load(
                     A.ck_vd + ((int64_t)(cn - 1) * BN + jn) * K + pos.sub * KT), ckd);
                 ckv = __ldcs(A.ck_vs + (int64_t)(cn - 1) * BN + jn);
             }
 
-            // recompute the chunk, keeping V^d and V^s of every step (and the Gaussians)
-            float vdh[L][KT];
-            float vsh[L];
-            float gsc[L];
-            float eh[KEEP_E ? L : 1][KTb];
+            // recompute the chunk, keeping V^d and V^s of every step (in registers for a
+            // single chunk, in shared memory, one slot per thread and step, otherwise)
+            typename AR::St vdh[MULTI ? 1 : L];
+            float vsh[MULTI ? 1 : L];
+            float gsc[MULTI ? 1 : L];     // single chunk: grad_spikes taken during the recompute
             {
-                float vd[KT];
-#pragma unroll
-                for (int k = 0; k < KT; ++k) vd[k] = vd0[k];
+                typename AR::St vd = vd0;
                 float v = v0;
                 bool s = (!MULTI || c == 0) ? false : (v0 >= P.theta);
+                const XT *xa = xrow + (int64_t)(t0 + H) * sX;      // this chunk, H steps ahead
+                const XT *xnn = xn;                                 // next chunk, from its start
 #pragma unroll
                 for (int tt = 0; tt < L; ++tt) {
                     float xv[KT];
-                    V::unpack(xb[tt], xv);
-                    gsc[tt] = S1::unpack(gsb[tt]);
-                    // refill slot tt for the next unit right after its value is taken
-                    if (has_next && tn + tt < T) {
-                        xb[tt] = V::load(xn + tt * stepX);
-                        gsb[tt] = S1::load(gsn + tt * BN);
+                    V::unpack(xb[tt % H], xv);
+                    if constexpr (!MULTI) {
+                        gsc[MULTI ? 0 : tt] = S1::unpack(gsb[tt]);
+                        if (tt < nnext) gsb[tt] = S1::load(gsn + (int64_t)tt * BN);
                     }
-                    if (t0 + tt < T) {
-                        float eb[KTb];
-                        const float z = lanes_sum<LPN>(
-                            dendrite_step<KT, G, PSI>(lp, vd, xv, P.residual != 0, inv_k, eb));
+                    // refill the slot with the step H ahead: later in this chunk, or the
+                    // first steps of the next chunk
+                    if (tt + H < L) {
+                        if (tt + H < ncur) xb[tt % H] = V::load(xa);
+                        xa += sX;
+                    } else {
+                        if (tt + H - L < nnext) xb[tt % H] = V::load(xnn);
+                        xnn += sX;
+                    }
+                    if (tt < ncur) {
+                        const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
                         v = soma_charge(z, v, s, P);
                         s = v >= P.theta;
-#pragma unroll
-                        for (int k = 0; k < KT; ++k) vdh[tt][k] = vd[k];
-                        vsh[tt] = v;
-                        if constexpr (KEEP_E) {
-#pragma unroll
-                            for (int b = 0; b < KTb; ++b) eh[KEEP_E ? tt : 0][b] = eb[b];
+                        if constexpr (MULTI) {
+                            float vda[KT];
+                            AR::to_array(vd, vda);
+                            hist[tt * kThreads + threadIdx.x] = Vec<float, KT>::pack(vda);
+                            hist_vs[tt * kThreads + threadIdx.x] = v;
+                        } else {
+                            vdh[MULTI ? 0 : tt] = vd;
+                            vsh[MULTI ? 0 : tt] = v;
                         }
                     }
                 }
             }
             // reverse-time recursion over the chunk
+            XT *gxp = gxrow + (int64_t)(t0 + L - 1) * sX;
+            const float *gvp = gvrow ? gvrow + (int64_t)(t0 + L - 1) * BN : nullptr;
 #pragma unroll
             for (int tt = L - 1; tt >= 0; --tt) {
-                const int t = t0 + tt;
-                if (t < T) {
-                    const float vs = vsh[tt];
+                float gs_t;
+                if constexpr (MULTI) {
+                    gs_t = S1::unpack(gsb[tt]);
+                    // refill slot tt with the next chunk's grad_spikes once this one is taken
+                    if (tt < nnext) gsb[tt] = S1::load(gsn + (int64_t)tt * BN);
+                } else {
+                    gs_t = gsc[MULTI ? 0 : tt];
+                }
+                if (tt < ncur) {
+                    float vs;
+                    typename AR::St vdt, vdp;                       // V^d[t], V^d[t-1]
+                    if constexpr (MULTI) {
+                        vs = hist_vs[tt * kThreads + threadIdx.x];
+                        float a[KT];
+                        Vec<float, KT>::unpack(hist[tt * kThreads + threadIdx.x], a);
+                        AR::from_array(vdt, a);
+                        if (tt > 0) {
+                            Vec<float, KT>::unpack(hist[(tt > 0 ? tt - 1 : 0) * kThreads + threadIdx.x], a);
+                            AR::from_array(vdp, a);
+                        } else {
+                            vdp = vd0;
+                        }
+                    } else {
+                        vs = vsh[MULTI ? 0 : tt];
+                        vdt = vdh[MULTI ? 0 : tt];
+                        vdp = (tt > 0) ? vdh[MULTI ? 0 : (tt > 0 ? tt - 1 : 0)] : vd0;
+                    }
                     const bool st = vs >= P.theta;
                     const float dvds = P.detach ? 0.f : (P.soft ? soft_dvds : __fmul_rn(hard_dvds, vs));
                     const float dvdv = (P.soft || !st) ? P.beta : 0.f;   // beta (1 - S[t]) when hard
-                    const float ds = __fmaf_rn(dvds, dvn, gsc[tt]);                      // dL/dS[t]
+                    const float ds = __fmaf_rn(dvds, dvn, gs_t);                          // dL/dS[t]
                     float dv = __fmaf_rn(surrogate(__fsub_rn(vs, P.theta)), ds,
                                          __fmul_rn(dvdv, dvn));                          // dL/dV^s[t]
-                    if (A.gv) dv = __fadd_rn(dv, __ldcs(A.gv + t * BN + j));
-                    float eb[KTb];
-                    if constexpr (KEEP_E) {
-#pragma unroll
-                        for (int b = 0; b < KTb; ++b) eb[b] = eh[KEEP_E ? tt : 0][b];
-                    } else if constexpr (PSI == PSI_MEXHAT) {
-#pragma unroll
-                        for (int b = 0; b < KTb; ++b) {
-                            float ss = 0.f;
-#pragma unroll
-                            for (int q = 0; q < G; ++q) {
-                                const float u = affine(lp, vdh[tt][b * G + q], b * G + q);
-                                ss = (q == 0) ? __fmul_rn(u, u) : __fmaf_rn(u, u, ss);
-                            }
-                            eb[b] = gauss_half(ss);
-                        }
-                    }
-                    float direct[KT];
-                    branch_backward<KT, G, PSI>(lp, vdh[tt], eb, dv, direct, acc);
+                    if (gvp) dv = __fadd_rn(dv, __ldcs(gvp));
                     float gxv[KT];
-                    const float res = P.residual ? __fmul_rn(dv, inv_k) : 0.f;
-#pragma unroll
-                    for (int k = 0; k < KT; ++k) {
-                        Ad[k] = __fmaf_rn(lp.a[k], Ad[k], direct[k]);
-                        gxv[k] = __fadd_rn(Ad[k], res);
-                        const float vprev = (tt > 0) ? vdh[tt > 0 ? tt - 1 : 0][k] : vd0[k];
-                        acc.ga[k] = __fmaf_rn(Ad[k], vprev, acc.ga[k]);
-                    }
-                    if (pos.active) V::store(gxr + t * stepX, gxv);
+                    AR::backward(lp, vdt, vdp, dv, Ad, acc, residual ? __fmul_rn(dv, inv_k) : 0.f, gxv);
+                    if (pos.active) V::store(gxp, gxv);
                     dvn = dv;
                 }
+                gxp -= sX;
+                if (gvp) gvp -= BN;
             }
         }
+        xrow += rX;
+        gsrow += jstep;
+        gxrow += rX;
+        if (gvrow) gvrow += jstep;
+        j += jstep;
     }
 
     // ---- parameter-gradient partials: per channel, fixed summation order
     float v[NA];
+    AR::acc_export(acc, v);
 #pragma unroll
-    for (int i = 0; i < KT; ++i) {
-        v[i] = (pos.active && !P.stateless) ? acc.ga[i] : 0.f;
-        v[KT + i] = pos.active ? acc.gxi[i] : 0.f;
-    }
-#pragma unroll
-    for (int b = 0; b < KTb; ++b) {
-        v[2 * KT + b] = pos.active ? acc.gz[b] : 0.f;
-        v[2 * KT + KTb + b] = pos.active ? acc.gk[b] : 0.f;
-    }
+    for (int a = 0; a < NA; ++a)
+        if (!pos.active || (a < KT && P.stateless)) v[a] = 0.f;
     // stage 1: within a warp, columns of one channel come in aligned runs of g.seg
     for (int d = 1; d < g.seg; d <<= 1) {
 #pragma unroll
         for (int a = 0; a < NA; ++a)
             v[a] = __fadd_rn(v[a], __shfl_xor_sync(0xffffffffu, v[a], d * LPN));
     }
-    // stage 2: run leaders meet in shared memory; red[a][tid]
-    extern __shared__ float red[];
+    // stage 2: run leaders meet in shared memory; red[a][tid] (reuses the history space)
+    float *red = reinterpret_cast<float *>(smem_f4);
+    __syncthreads();
 #pragma unroll
     for (int a = 0; a < NA; ++a) red[a * kThreads + threadIdx.x] = v[a];
     __syncthreads();
@@ -683,7 +869,9 @@ template <int K, int G, int PSI, int XT, int L>
 cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
     using T = typename XType<XT>::type;
     constexpr int KT = (K < 4) ? K : 4;
-    const size_t smem = sizeof(float) * acc_count<KT, G>() * kThreads;
+    const size_t red = sizeof(float) * acc_count<KT, G>() * kThreads;
+    const size_t hist = (L > 4) ? sizeof(float) * (KT + 1) * L * kThreads : 0;
+    const size_t smem = red > hist ? red : hist;
     dendsn_backward_kernel<K, G, PSI, T, L><<<blocks, kThreads, smem, s>>>(a);
     return cudaGetLastError();
 }
