@@ -517,16 +517,41 @@ __device__ __forceinline__ ThreadPos thread_pos(const Geometry &g) {
 }
 
 // ---------------------------------------------------------------- forward
+// Tuning: the forward's minimum resident blocks per SM (register cap), and whether
+// its inputs are staged through shared memory with cp.async (else a register ring).
+#ifndef DENDSN_FWD_MINB
+#define DENDSN_FWD_MINB 3
+#endif
+#ifndef DENDSN_FWD_ASYNC
+#define DENDSN_FWD_ASYNC 1
+#endif
+constexpr int kFwdDepth = 8;   // steps of x in flight per thread on the cp.async path
+
+// Asynchronous 4/8/16-byte global -> shared copy (PTX cp.async). `dep` is an unused
+// operand that orders the copy after the computation producing it.
+template <int BYTES>
+__device__ __forceinline__ void cp_async(void *smem, const void *gmem, float dep) {
+    const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem);
+    if constexpr (BYTES == 16)
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16; // %2\n" :: "r"(d), "l"(gmem), "f"(dep) : "memory");
+    else
+        asm volatile("cp.async.ca.shared.global [%0], [%1], %3; // %2\n" :: "r"(d), "l"(gmem), "f"(dep), "n"(BYTES) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" :: "n"(N) : "memory"); }
+
 // x is prefetched kFwdBatch steps ahead of use (a ring of kFwdBatch registers);
 // checkpoints every g.L steps (g.L is a power of two and a multiple of the batch).
 template <int K, int G, int PSI, typename XT>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, DENDSN_FWD_MINB)
 dendsn_forward_kernel(const FwdArgs A) {
     constexpr int KT = (K < 4) ? K : 4;
     constexpr int LPN = K / KT;
     constexpr int L = kFwdBatch;
     using V = Vec<XT, KT>;
     using AR = Arith<KT, G, PSI>;
+    constexpr bool ASYNC = DENDSN_FWD_ASYNC && sizeof(typename V::Raw) >= 4;
     const Geometry &g = A.g;
     const Params &P = A.p;
     const ThreadPos pos = thread_pos<LPN>(g);
@@ -547,6 +572,69 @@ dendsn_forward_kernel(const FwdArgs A) {
     const bool write_ck = (A.ck_vd != nullptr) && g.n_ck > 0 && pos.active;
     const bool store = pos.active && pos.sub == 0;
     const bool residual = P.residual != 0;
+
+    if constexpr (ASYNC) {
+        // Inputs are staged through a ring of kFwdDepth shared-memory slots per thread,
+        // filled by cp.async kFwdDepth steps ahead of use along this thread's
+        // (row, step) sequence; each thread reads only its own slots.
+        constexpr int D = kFwdDepth;
+        using Raw = typename V::Raw;
+        extern __shared__ float4 fwd_smem[];
+        Raw *ring = reinterpret_cast<Raw *>(fwd_smem) + threadIdx.x;     // slot k at ring[k * kThreads]
+        const XT *ip = xrow;                    // next step to fetch
+        int it = 0, ir = 0;                     // its step and row
+        const int64_t row_jump = rX - (int64_t)T * sX;
+#pragma unroll
+        for (int k = 0; k < D; ++k) {
+            if (ir < pos.nrows) cp_async<sizeof(Raw)>(ring + k * kThreads, ip, 0.f);
+            cp_async_commit();
+            ip += sX;
+            if (++it == T) { it = 0; ++ir; ip += row_jump; }
+        }
+        int slot = 0;
+        int64_t j = j0;
+        for (int i = 0; i < pos.nrows; ++i) {
+            if (P.mask_mode == 2) AR::neuron_mask(P, g, j % g.N, pos.chan, pos.sub, lp);
+            typename AR::St vd;
+            AR::zero(vd);
+            float v = 0.f;
+            bool s = false;
+            XT *sp = srow;
+            float *vp = vrow;
+            for (int t = 0; t < T; ++t) {
+                cp_async_wait<D - 1>();
+                float xv[KT];
+                V::unpack(ring[slot * kThreads], xv);
+                const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
+                // the slot's value has been used (z depends on it): refill it
+                if (ir < pos.nrows) cp_async<sizeof(Raw)>(ring + slot * kThreads, ip, z);
+                cp_async_commit();
+                ip += sX;
+                if (++it == T) { it = 0; ++ir; ip += row_jump; }
+                v = soma_charge(z, v, s, P);
+                s = v >= P.theta;                          // Eq. methods-lif-fire
+                if (store) {
+                    Scalar<XT>::store_spike(sp, s);
+                    if (vp) __stcs(vp, v);
+                }
+                sp += BN;
+                if (vp) vp += BN;
+                if (write_ck && ((t + 1) & (g.L - 1)) == 0 && t + 1 < T) {
+                    const int ck = (t + 1) / g.L - 1;
+                    float vda[KT];
+                    AR::to_array(vd, vda);
+                    Vec<float, KT>::store(A.ck_vd + ((int64_t)ck * BN + j) * K + pos.sub * KT, vda);
+                    if (pos.sub == 0) __stcs(A.ck_vs + (int64_t)ck * BN + j, v);
+                }
+                slot = (slot == D - 1) ? 0 : slot + 1;
+            }
+            srow += jstep;
+            if (vrow) vrow += jstep;
+            j += jstep;
+        }
+        cp_async_wait<0>();
+        return;
+    }
 
     typename V::Raw xb[L];
     {
@@ -861,7 +949,10 @@ dendsn_backward_kernel(const BwdArgs A) {
 template <int K, int G, int PSI, int XT>
 cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s) {
     using T = typename XType<XT>::type;
-    dendsn_forward_kernel<K, G, PSI, T><<<blocks, kThreads, 0, s>>>(a);
+    constexpr int KT = (K < 4) ? K : 4;
+    constexpr size_t raw = sizeof(typename Vec<T, KT>::Raw);
+    const size_t smem = (DENDSN_FWD_ASYNC && raw >= 4) ? raw * kFwdDepth * kThreads : 0;
+    dendsn_forward_kernel<K, G, PSI, T><<<blocks, kThreads, smem, s>>>(a);
     return cudaGetLastError();
 }
 
