@@ -526,6 +526,10 @@ __device__ __forceinline__ ThreadPos thread_pos(const Geometry &g) {
 #define DENDSN_FWD_ASYNC 1
 #endif
 constexpr int kFwdDepth = 8;   // steps of x in flight per thread on the cp.async path
+#ifndef DENDSN_BWD_ASYNC
+#define DENDSN_BWD_ASYNC 1
+#endif
+constexpr int kBwdDepth = 8;   // steps of x in flight per thread in the backward's cp.async ring
 
 // Asynchronous 4/8/16-byte global -> shared copy (PTX cp.async). `dep` is an unused
 // operand that orders the copy after the computation producing it.
@@ -714,6 +718,11 @@ dendsn_backward_kernel(const BwdArgs A) {
     using S1 = Scalar<XT>;
     using AR = Arith<KT, G, PSI>;
     using HistRaw = typename Vec<float, KT>::Raw;
+    using XRaw = typename V::Raw;
+    // multi-chunk: x staged through a per-thread cp.async ring in shared memory; single
+    // chunk (T <= 4): a register ring, which measured faster there
+    constexpr bool BASYNC = DENDSN_BWD_ASYNC && MULTI && sizeof(XRaw) >= 4;
+    constexpr int D = kBwdDepth;
     const Geometry &g = A.g;
     const Params &P = A.p;
     const ThreadPos pos = thread_pos<LPN>(g);
@@ -738,11 +747,36 @@ dendsn_backward_kernel(const BwdArgs A) {
     extern __shared__ float4 smem_f4[];
     HistRaw *hist = reinterpret_cast<HistRaw *>(smem_f4);                             // [L][kThreads]
     float *hist_vs = reinterpret_cast<float *>(hist + (MULTI ? L * kThreads : 0));   // [L][kThreads]
+    XRaw *xring = reinterpret_cast<XRaw *>(hist_vs + (MULTI ? L * kThreads : 0)) + threadIdx.x;   // [D][kThreads]
+    // cp.async walker over this thread's sequence: rows, chunks in reverse, steps forward
+    const XT *const xbase = xrow;
+    int wr = 0, wc = nc - 1, wt = 0;
+    int wlen = min(L, T - wc * L);
+    const XT *wp = xbase + (int64_t)wc * L * sX;
+    auto walk = [&]() {
+        if (++wt == wlen) {
+            wt = 0;
+            if (--wc < 0) { wc = nc - 1; ++wr; }
+            wlen = min(L, T - wc * L);
+            wp = xbase + wr * rX + (int64_t)wc * L * sX;
+        } else {
+            wp += sX;
+        }
+    };
+    int xslot = 0;
+    if constexpr (BASYNC) {
+#pragma unroll
+        for (int k = 0; k < D; ++k) {
+            if (wr < pos.nrows) cp_async<sizeof(XRaw)>(xring + k * kThreads, wp, 0.f);
+            cp_async_commit();
+            walk();
+        }
+    }
 
     typename AR::Acc acc;
     AR::acc_zero(acc);
 
-    typename V::Raw xb[H];            // x of the next H steps to recompute
+    XRaw xb[BASYNC ? 1 : H];          // register ring: x of the next H steps to recompute
     typename S1::Raw gsb[L];          // grad_spikes of the current chunk
     float ckd[KT];                    // checkpoint V^d entering the current chunk
     float ckv = 0.f;                  // checkpoint V^s entering the current chunk
@@ -755,7 +789,7 @@ dendsn_backward_kernel(const BwdArgs A) {
 #pragma unroll
         for (int tt = 0; tt < L; ++tt) {
             if (t0 + tt < T) {
-                if (tt < H) xb[tt < H ? tt : 0] = V::load(p);
+                if (!BASYNC && tt < H) xb[(!BASYNC && tt < H) ? tt : 0] = V::load(p);
                 gsb[tt] = S1::load(q);
             }
             p += sX;
@@ -814,22 +848,35 @@ dendsn_backward_kernel(const BwdArgs A) {
 #pragma unroll
                 for (int tt = 0; tt < L; ++tt) {
                     float xv[KT];
-                    V::unpack(xb[tt % H], xv);
+                    if constexpr (!BASYNC) V::unpack(xb[BASYNC ? 0 : tt % H], xv);
                     if constexpr (!MULTI) {
                         gsc[MULTI ? 0 : tt] = S1::unpack(gsb[tt]);
                         if (tt < nnext) gsb[tt] = S1::load(gsn + (int64_t)tt * BN);
                     }
-                    // refill the slot with the step H ahead: later in this chunk, or the
-                    // first steps of the next chunk
-                    if (tt + H < L) {
-                        if (tt + H < ncur) xb[tt % H] = V::load(xa);
-                        xa += sX;
-                    } else {
-                        if (tt + H - L < nnext) xb[tt % H] = V::load(xnn);
-                        xnn += sX;
+                    if constexpr (!BASYNC) {
+                        // refill the slot with the step H ahead: later in this chunk, or
+                        // the first steps of the next chunk
+                        if (tt + H < L) {
+                            if (tt + H < ncur) xb[BASYNC ? 0 : tt % H] = V::load(xa);
+                            xa += sX;
+                        } else {
+                            if (tt + H - L < nnext) xb[BASYNC ? 0 : tt % H] = V::load(xnn);
+                            xnn += sX;
+                        }
                     }
                     if (tt < ncur) {
+                        if constexpr (BASYNC) {
+                            cp_async_wait<D - 1>();
+                            V::unpack(xring[xslot * kThreads], xv);
+                        }
                         const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
+                        if constexpr (BASYNC) {
+                            // the slot's value has been used (z depends on it): refill it
+                            if (wr < pos.nrows) cp_async<sizeof(XRaw)>(xring + xslot * kThreads, wp, z);
+                            cp_async_commit();
+                            walk();
+                            xslot = (xslot == D - 1) ? 0 : xslot + 1;
+                        }
                         v = soma_charge(z, v, s, P);
                         s = v >= P.theta;
                         if constexpr (MULTI) {
@@ -913,6 +960,7 @@ dendsn_backward_kernel(const BwdArgs A) {
     }
     // stage 2: run leaders meet in shared memory; red[a][tid] (reuses the history space)
     float *red = reinterpret_cast<float *>(smem_f4);
+    if constexpr (BASYNC) cp_async_wait<0>();
     __syncthreads();
 #pragma unroll
     for (int a = 0; a < NA; ++a) red[a * kThreads + threadIdx.x] = v[a];
@@ -946,12 +994,21 @@ dendsn_backward_kernel(const BwdArgs A) {
 }
 
 // ---------------------------------------------------------------- launchers
+// Dynamic shared memory above 48 KB needs an explicit opt-in per kernel.
+template <typename Kern>
+cudaError_t allow_smem(Kern kernel, size_t bytes) {
+    if (bytes <= 48 * 1024) return cudaSuccess;
+    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+}
+
 template <int K, int G, int PSI, int XT>
 cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s) {
     using T = typename XType<XT>::type;
     constexpr int KT = (K < 4) ? K : 4;
     constexpr size_t raw = sizeof(typename Vec<T, KT>::Raw);
     const size_t smem = (DENDSN_FWD_ASYNC && raw >= 4) ? raw * kFwdDepth * kThreads : 0;
+    cudaError_t e = allow_smem(dendsn_forward_kernel<K, G, PSI, T>, smem);
+    if (e != cudaSuccess) return e;
     dendsn_forward_kernel<K, G, PSI, T><<<blocks, kThreads, smem, s>>>(a);
     return cudaGetLastError();
 }
@@ -962,7 +1019,11 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
     constexpr int KT = (K < 4) ? K : 4;
     const size_t red = sizeof(float) * acc_count<KT, G>() * kThreads;
     const size_t hist = (L > 4) ? sizeof(float) * (KT + 1) * L * kThreads : 0;
-    const size_t smem = red > hist ? red : hist;
+    constexpr size_t xraw = sizeof(typename Vec<T, KT>::Raw);
+    const size_t ring = (DENDSN_BWD_ASYNC && L > 4 && xraw >= 4) ? xraw * kBwdDepth * kThreads : 0;
+    const size_t smem = red > hist + ring ? red : hist + ring;
+    cudaError_t e = allow_smem(dendsn_backward_kernel<K, G, PSI, T, L>, smem);
+    if (e != cudaSuccess) return e;
     dendsn_backward_kernel<K, G, PSI, T, L><<<blocks, kThreads, smem, s>>>(a);
     return cudaGetLastError();
 }
