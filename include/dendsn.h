@@ -133,6 +133,32 @@ dendsn_status dendsn_backward(const dendsn_config *cfg, const void *x, const flo
                               float *grad_alpha, float *grad_xi, float *grad_zeta,
                               float *grad_kappa, void *scratch, void *stream);
 
+/*
+ * Same computation and outputs as dendsn_backward, without the caller's scratch buffer:
+ * for callers that cannot allocate device memory for it, such as a C host that only
+ * receives device pointers for the layer's tensors, or a runtime whose device memory is
+ * budgeted in advance and that must not allocate per call. (The paper has no
+ * counterpart; this is an interface convenience.)
+ *   - The parameter-gradient partials go to a buffer compiled into the library:
+ *     8 MiB of device memory on every GPU that loads the library, held until the
+ *     process exits. A layer whose dendsn_workspace_size scratch_bytes exceeds 8 MiB
+ *     is rejected with DENDSN_ERR_UNSUPPORTED before anything is enqueued.
+ *   - The first call on a device looks up that buffer's device address (with that
+ *     device current) and caches it; make that first call before any stream capture.
+ *   - All calls share the one buffer, which keeps the last call's contents. Nothing in
+ *     it needs to start at zero. Calls whose executions overlap on the GPU (for example
+ *     on two streams without ordering between them) race on it and give wrong results.
+ *   - Allocates nothing: no cudaMalloc, cudaFree or allocating library call.
+ * Arguments are those of dendsn_backward minus `scratch`.
+ */
+dendsn_status dendsn_backward_noalloc(const dendsn_config *cfg, const void *x,
+                                      const float *alpha, const float *xi, const float *zeta,
+                                      const float *kappa, const uint8_t *mask,
+                                      const void *grad_spikes, const float *grad_v,
+                                      const void *saved, void *grad_x, float *grad_alpha,
+                                      float *grad_xi, float *grad_zeta, float *grad_kappa,
+                                      void *stream);
+
 /* Static description of a status code. */
 const char *dendsn_status_string(dendsn_status status);
 

@@ -145,6 +145,29 @@ def dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, s
         _stream(stream)))
 
 
+_noalloc_ready = False
+
+
+def dendsn_backward_noalloc(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved,
+                            grad_x, grad_alpha, grad_xi, grad_zeta, grad_kappa, stream=None):
+    """dendsn_backward without a scratch buffer (the library's built-in 8 MiB one).
+
+    For callers that cannot allocate device scratch memory per call; see the header
+    for the sharing rules of the built-in buffer.
+    """
+    global _noalloc_ready
+    lib = load()
+    if not _noalloc_ready:
+        lib.dendsn_backward_noalloc.argtypes = [ctypes.POINTER(dendsn_config)] + \
+            [ctypes.c_void_p] * 15
+        lib.dendsn_backward_noalloc.restype = ctypes.c_int
+        _noalloc_ready = True
+    _check("dendsn_backward_noalloc", lib.dendsn_backward_noalloc(
+        ctypes.byref(cfg), _ptr(x), _ptr(alpha), _ptr(xi), _ptr(zeta), _ptr(kappa),
+        _ptr(mask), _ptr(grad_spikes), _ptr(grad_v), _ptr(saved), _ptr(grad_x),
+        _ptr(grad_alpha), _ptr(grad_xi), _ptr(grad_zeta), _ptr(grad_kappa), _stream(stream)))
+
+
 # ------------------------------------------------------------------ tensor-level helpers
 def _xdtype(cfg) -> torch.dtype:
     return torch.bfloat16 if cfg.x_dtype == BF16 else torch.float32

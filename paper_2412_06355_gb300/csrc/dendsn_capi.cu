@@ -2,6 +2,7 @@
 // kernel instances, and the deterministic parameter-gradient finalize kernel.
 #include <algorithm>
 #include <atomic>
+#include <mutex>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -351,3 +352,65 @@ const char *dendsn_last_error(void) { return g_last_error; }
 uint64_t dendsn_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------- scratch-free backward
+// A backward for callers that cannot hand the library a scratch buffer: for example a
+// plain C host that only receives device pointers for the tensors and has no device
+// allocator of its own, or a runtime whose device memory is budgeted up front and that
+// must not allocate on each call. The per-block parameter-gradient partials go to a
+// fixed buffer compiled into the library instead of caller memory.
+namespace {
+
+// Capacity of the built-in scratch buffer. Every GPU that loads the library keeps this
+// much device memory reserved until the process exits.
+constexpr size_t kNoAllocScratchBytes = size_t(8) << 20;   // 8 MiB
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+constexpr int kMaxDevices = 256;
+std::mutex g_noalloc_mutex;
+void *g_noalloc_ptr[kMaxDevices] = {};   // device address of g_noalloc_scratch, per device
+
+// Device address of the built-in buffer on the current device. The first call on a
+// device looks it up (cudaGetSymbolAddress, with that device current) and caches it.
+dendsn_status noalloc_scratch(void **out) {
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess)
+        return fail(DENDSN_ERR_CUDA, "cudaGetDevice failed: %s", cudaGetErrorString(e));
+    if (dev < 0 || dev >= kMaxDevices)
+        return fail(DENDSN_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (g_noalloc_ptr[dev] == nullptr) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || p == nullptr)
+            return fail(DENDSN_ERR_CUDA, "cudaGetSymbolAddress of the built-in scratch failed: %s",
+                        cudaGetErrorString(e));
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = g_noalloc_ptr[dev];
+    return DENDSN_OK;
+}
+
+}  // namespace
+
+extern "C" dendsn_status dendsn_backward_noalloc(
+    const dendsn_config *cfg, const void *x, const float *alpha, const float *xi,
+    const float *zeta, const float *kappa, const uint8_t *mask, const void *grad_spikes,
+    const float *grad_v, const void *saved, void *grad_x, float *grad_alpha, float *grad_xi,
+    float *grad_zeta, float *grad_kappa, void *stream) {
+    Plan pl;
+    dendsn_status st = make_plan(cfg, &pl, true);
+    if (st != DENDSN_OK) return st;
+    if (pl.scratch_bytes > kNoAllocScratchBytes)
+        return fail(DENDSN_ERR_UNSUPPORTED,
+                    "this layer needs %zu bytes of scratch, more than the %zu-byte built-in "
+                    "buffer of dendsn_backward_noalloc; use dendsn_backward with a caller buffer",
+                    pl.scratch_bytes, kNoAllocScratchBytes);
+    void *scratch = nullptr;
+    if ((st = noalloc_scratch(&scratch)) != DENDSN_OK) return st;
+    // Nothing in the buffer needs to start at zero: the backward kernel writes every
+    // partial sum that the finalize kernel then reads, in the same call.
+    return dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved,
+                           grad_x, grad_alpha, grad_xi, grad_zeta, grad_kappa, scratch, stream);
+}

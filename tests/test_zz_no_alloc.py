@@ -1,0 +1,78 @@
+"""The scratch-free backward (dendsn_backward_noalloc) against dendsn_backward.
+
+Some callers cannot give the library a device scratch buffer (a C host that only holds
+device pointers for the tensors, or a runtime that must not allocate per call); for them
+the library keeps its own fixed buffer. These checks call both entry points through the
+C ABI on the same inputs and require the same gradients, within the parity tolerances,
+on two calls in a row with different layer sizes, so that what the first call leaves in
+the shared buffer cannot leak into the second. This file sorts last so that a run that
+stops at its first failure has already run every other test; it also passes on its own
+in a fresh process (the first call on the device performs the one-time set-up).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2412_06355_gb300 import binding, workloads
+
+from parity import BF16_ATOL_REL, BF16_RTOL, G_ATOL_REL, G_RTOL, assert_close, to_dev
+
+pytestmark = pytest.mark.gpu
+
+CASES = [
+    # large first (a transformer-token layer: per-neuron mask, many channels) ...
+    workloads.scaled(workloads.WORKLOADS["token_dbg"], B=4),
+    # ... then a smaller conv-shaped layer with checkpoints and bf16 inputs
+    workloads.Workload("small", T=12, B=3, N=2 * 256, K=8, G=1, C=2, inner=256, dtype="bf16",
+                       psi="mh", reset="soft", seed=77),
+]
+
+
+def run_both(w):
+    cfg = binding.config_of(w)
+    inp = to_dev(workloads.make_inputs(w, "cpu", with_gv=True))
+    saved, scratch = binding.workspace(cfg)
+    binding.forward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"],
+                    inp["mask"], saved=saved)
+    ref = binding.backward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"],
+                           inp["mask"], inp["gs"], inp["gv"], saved, scratch)
+    C, K, Kb = cfg.C, cfg.K, cfg.K // cfg.G
+    got = dict(gx=torch.full_like(inp["x"], float("nan")),
+               galpha=torch.full((C, K), float("nan"), device="cuda"),
+               gxi=torch.full((C, K), float("nan"), device="cuda"),
+               gzeta=torch.full((C, Kb), float("nan"), device="cuda"),
+               gkappa=torch.full((C, Kb), float("nan"), device="cuda"))
+    binding.dendsn_backward_noalloc(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"],
+                                    inp["kappa"], inp["mask"], inp["gs"], inp["gv"], saved,
+                                    got["gx"], got["galpha"], got["gxi"], got["gzeta"],
+                                    got["gkappa"])
+    torch.cuda.synchronize()
+    return w, {k: oracle.to_f64(v) for k, v in ref.items()}, {k: oracle.to_f64(v) for k, v in got.items()}
+
+
+def test_noalloc_backward_matches_backward_twice_in_a_row():
+    if not torch.cuda.is_available():
+        pytest.fail("needs a CUDA device")
+    for w in CASES:
+        w, ref, got = run_both(w)
+        rt, ar = (BF16_RTOL, BF16_ATOL_REL) if w.dtype == "bf16" else (G_RTOL, G_ATOL_REL)
+        assert_close(f"{w.name} grad_x", got["gx"], ref["gx"], rt, ar)
+        for k in ("galpha", "gxi", "gzeta", "gkappa"):
+            assert_close(f"{w.name} {k}", got[k], ref[k], G_RTOL, G_ATOL_REL)
+
+
+def test_noalloc_rejects_layers_beyond_its_buffer():
+    if not torch.cuda.is_available():
+        pytest.fail("needs a CUDA device")
+    # 65536 channels of one neuron each: every block touches 33 channels, and the
+    # per-block partials need 8.25 MiB, just over the built-in 8 MiB
+    w = workloads.Workload("huge", T=1, B=32, N=65536, K=4, G=1, C=65536, inner=1,
+                           dtype="f32", psi="mh", reset="hard")
+    cfg = binding.config_of(w)
+    _, need = binding.dendsn_workspace_size(cfg)
+    assert need > 8 << 20
+    d = torch.empty(16, device="cuda")
+    with pytest.raises(binding.DendSNError) as e:
+        binding.dendsn_backward_noalloc(cfg, d, d, d, d, d, None, d, None, None, d, d, d, d, d)
+    assert e.value.status == 2 and "8388608" in str(e.value)
