@@ -10,6 +10,7 @@ restatement and invariants; see tests/test_oracle_pins.py).
 """
 from __future__ import annotations
 
+import contextlib
 import ctypes
 import dataclasses
 import os
@@ -66,17 +67,36 @@ def build(force: bool = False) -> str:
     return _LIB_PATH
 
 
+def _configure(lib):
+    P = ctypes.c_void_p
+    for name, nargs in (("oracle_forward", 11), ("oracle_backward", 16)):
+        fn = getattr(lib, name)
+        fn.restype = ctypes.c_int
+        fn.argtypes = [ctypes.POINTER(_Cfg)] + [P] * (nargs - 1)
+    return lib
+
+
 def _load():
     global _lib
     if _lib is None:
-        lib = ctypes.CDLL(build())
-        P = ctypes.c_void_p
-        for name, nargs in (("oracle_forward", 11), ("oracle_backward", 16)):
-            fn = getattr(lib, name)
-            fn.restype = ctypes.c_int
-            fn.argtypes = [ctypes.POINTER(_Cfg)] + [P] * (nargs - 1)
-        _lib = lib
+        _lib = _configure(ctypes.CDLL(build()))
     return _lib
+
+
+@contextlib.contextmanager
+def using_library(path: str):
+    """Test hook: run this wrapper against another build of the oracle (a mutant)."""
+    global _lib
+    saved = _lib
+    _lib = _configure(ctypes.CDLL(path))
+    try:
+        yield
+    finally:
+        _lib = saved
+
+
+def source_path() -> str:
+    return _SRC
 
 
 def to_f64(a) -> np.ndarray:
