@@ -284,7 +284,7 @@ def run_reference(args):
 def run_ours(args):
     import torch
     import torch.distributed as dist
-    from paper_2412_06355_gb300 import binding, workloads
+    from paper_2412_06355_gb300 import binding, distributed, workloads
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -305,8 +305,8 @@ def run_ours(args):
     saved, scratch = binding.workspace(cfg, dev)
     spikes = torch.empty(x.shape[:3], dtype=x.dtype, device=dev)
     gx = torch.empty_like(x)
-    grads = torch.empty(2 * w.C * w.K + 2 * w.C * w.Kb, dtype=torch.float32, device=dev)
-    ga, gxi, gz, gk = torch.split(grads, [w.C * w.K, w.C * w.K, w.C * w.Kb, w.C * w.Kb])
+    grads, views = distributed.param_grad_buffer(w.C, w.K, w.Kb, dev)
+    ga, gxi, gz, gk = (views[k] for k in ("galpha", "gxi", "gzeta", "gkappa"))
     stream = torch.cuda.current_stream()
 
     def step(ev=None):
@@ -320,7 +320,7 @@ def run_ours(args):
         if ev is not None:
             ev[2].record(stream)
         if world > 1:
-            dist.all_reduce(grads)
+            distributed.sum_param_grads(grads)
 
     clocks = ClockSampler(dev.index)
     if rank == 0:
