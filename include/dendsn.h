@@ -41,7 +41,7 @@
  *    "Dendritic spiking neural networks", constraint 3). N must be a multiple of
  *    C * inner. A layer-wide decay alpha (the paper's choice) is passed as a [C, K]
  *    array of equal values; its gradient is the sum of grad_alpha.
- *  - Supported: K in {1, 2, 4, 8, 16}; G in {1, 2, 4} with G dividing min(K, 4);
+ *  - Supported: K in {1, 2, 4, 8, 16}; G in {1, 2, 4} with G dividing K;
  *    T >= 0; B * N < 2^31 * C * inner. Others return DENDSN_ERR_UNSUPPORTED.
  */
 #ifndef DENDSN_H

@@ -66,9 +66,8 @@ dendsn_status fail(dendsn_status st, const char *fmt, ...) {
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 struct Plan {
-    Geometry g;
-    int blocks;        // forward/backward grid
-    int LPN;
+    Geometry gf, gb;   // forward and backward tilings (block sizes may differ)
+    int blocks_f, blocks_b;
     size_t saved_bytes, scratch_bytes, ck_vd_bytes;
     int sx;            // bytes per x element
 };
@@ -87,6 +86,30 @@ int sm_count() {
 }
 
 bool is01(int32_t v) { return v == 0 || v == 1; }
+
+// Tiling of the O x P neuron matrix for blocks of nt threads, lpn lanes per neuron.
+dendsn_status tile(Geometry &g, int nt, int lpn, int64_t sms, int64_t *blocks) {
+    const int W = 32 / lpn;                     // columns per warp
+    const int full = nt / lpn;                  // columns of a one-row tile
+    g.TXn = (g.inner >= W && g.P % full == 0) ? full : W;
+    g.TY = nt / (g.TXn * lpn);
+    g.seg = (g.inner % W == 0) ? W : ((W % g.inner == 0) ? g.inner : 1);
+    g.nCT = (int32_t)((g.P + g.TXn - 1) / g.TXn);
+    // rows per thread: about 16 blocks per SM in total, at least one row
+    const int64_t target_blocks = 16LL * sms;
+    const int64_t rg_target = std::max<int64_t>(1, (target_blocks + g.nCT - 1) / g.nCT);
+    const int64_t rows_per_rg = std::max<int64_t>(1, (g.O + rg_target - 1) / rg_target);
+    g.R = (int32_t)std::max<int64_t>(1, (rows_per_rg + g.TY - 1) / g.TY);
+    const int64_t nRG = (g.O + (int64_t)g.R * g.TY - 1) / ((int64_t)g.R * g.TY);
+    g.nRG = (int32_t)nRG;
+    // channels one column tile touches (tiles start at multiples of TXn)
+    if (g.TXn % g.inner == 0) g.nch_max = g.TXn / g.inner;
+    else if (g.inner % g.TXn == 0) g.nch_max = 1;
+    else g.nch_max = std::min<int32_t>(g.C, (g.TXn - 1) / g.inner + 2);
+    *blocks = (int64_t)g.nCT * nRG;
+    if (*blocks > INT32_MAX) return fail(DENDSN_ERR_UNSUPPORTED, "grid too large");
+    return DENDSN_OK;
+}
 
 dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) {
     if (cfg == nullptr) return fail(DENDSN_ERR_INVALID_ARG, "cfg is NULL");
@@ -107,8 +130,8 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) 
     if (!std::isfinite(c.theta) || !std::isfinite(c.beta))
         return fail(DENDSN_ERR_INVALID_ARG, "theta and beta must be finite");
     const bool k_ok = c.K == 1 || c.K == 2 || c.K == 4 || c.K == 8 || c.K == 16;
-    const int KT = c.K < 4 ? c.K : 4;
-    if (!k_ok || KT % c.G != 0)
+    const int KT = lane_compartments(c.K);
+    if (!k_ok || c.G > 4 || KT % c.G != 0)
         return fail(DENDSN_ERR_UNSUPPORTED, "K=%d G=%d not compiled in", c.K, c.G);
     const int64_t P = (int64_t)c.C * c.inner;
     if (P > INT32_MAX) return fail(DENDSN_ERR_UNSUPPORTED, "C*inner too large");
@@ -119,11 +142,8 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) 
     const int64_t O = BN / P;
     if (O > INT32_MAX) return fail(DENDSN_ERR_UNSUPPORTED, "too many rows");
 
-    Geometry &g = pl->g;
+    Geometry g;
     std::memset(&g, 0, sizeof g);
-    const int LPN = c.K / KT;
-    const int W = 32 / LPN;                     // columns per warp
-    const int full = kThreads / LPN;            // columns of a one-row tile
     g.O = O;
     g.BN = BN;
     g.P = (int32_t)P;
@@ -133,27 +153,21 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) 
     g.T = c.T;
     g.K = c.K;
     g.Kb = c.K / c.G;
-    g.TXn = (c.inner >= W && P % full == 0) ? full : W;
-    g.TY = kThreads / (g.TXn * LPN);
-    g.seg = (c.inner % W == 0) ? W : ((W % c.inner == 0) ? c.inner : 1);
-    g.nCT = (int32_t)((P + g.TXn - 1) / g.TXn);
     g.L = (c.T <= 4) ? 4 : 8;
     g.n_ck = (c.T > g.L) ? (c.T + g.L - 1) / g.L - 1 : 0;
-    // rows per thread: about 16 blocks per SM in total, but at least one row
-    const int64_t target_blocks = 16LL * (need_sm_count ? sm_count() : 152);
-    const int64_t rg_target = std::max<int64_t>(1, (target_blocks + g.nCT - 1) / g.nCT);
-    const int64_t rows_per_rg = std::max<int64_t>(1, (O + rg_target - 1) / rg_target);
-    g.R = (int32_t)std::max<int64_t>(1, (rows_per_rg + g.TY - 1) / g.TY);
-    const int64_t nRG = (O + (int64_t)g.R * g.TY - 1) / ((int64_t)g.R * g.TY);
-    g.nRG = (int32_t)nRG;
-    g.nch_max = std::min<int32_t>(c.C, (g.TXn - 1) / c.inner + 2);
-    const int64_t blocks = (int64_t)g.nCT * nRG;
-    if (blocks > INT32_MAX) return fail(DENDSN_ERR_UNSUPPORTED, "grid too large");
-    pl->blocks = (int)blocks;
-    pl->LPN = LPN;
+    const int64_t sms = need_sm_count ? sm_count() : 152;
+    int64_t bf = 0, bb = 0;
+    pl->gf = g;
+    pl->gb = g;
+    const int KTB = bwd_lane_compartments(c.K, c.G, c.x_dtype, g.L);
+    dendsn_status st = tile(pl->gf, fwd_threads(c.K), c.K / KT, sms, &bf);
+    if (st != DENDSN_OK) return st;
+    if ((st = tile(pl->gb, bwd_threads(KTB), c.K / KTB, sms, &bb)) != DENDSN_OK) return st;
+    pl->blocks_f = (int)bf;
+    pl->blocks_b = (int)bb;
     pl->sx = (c.x_dtype == DENDSN_BF16) ? 2 : 4;
     const size_t NP = 2 * (size_t)c.K + 2 * (size_t)g.Kb;
-    pl->scratch_bytes = (size_t)blocks * g.nch_max * NP * sizeof(float);
+    pl->scratch_bytes = (size_t)bb * pl->gb.nch_max * NP * sizeof(float);
     pl->scratch_bytes = (pl->scratch_bytes + 15) / 16 * 16;
     pl->ck_vd_bytes = (size_t)g.n_ck * (size_t)BN * c.K * sizeof(float);
     pl->saved_bytes = pl->ck_vd_bytes + (size_t)g.n_ck * (size_t)BN * sizeof(float);
@@ -250,7 +264,7 @@ dendsn_status dendsn_forward(const dendsn_config *cfg, const void *x, const floa
     Plan pl;
     dendsn_status st = make_plan(cfg, &pl, true);
     if (st != DENDSN_OK) return st;
-    if (pl.g.BN == 0 || pl.g.T == 0) return DENDSN_OK;
+    if (pl.gf.BN == 0 || pl.gf.T == 0) return DENDSN_OK;
     if (!x || !spikes) return fail(DENDSN_ERR_INVALID_ARG, "x or spikes is NULL");
     if ((st = check_params(alpha, xi, zeta, kappa, mask)) != DENDSN_OK) return st;
     if (!aligned(x, 16)) return fail(DENDSN_ERR_MISALIGNED, "x must be 16-byte aligned");
@@ -258,15 +272,15 @@ dendsn_status dendsn_forward(const dendsn_config *cfg, const void *x, const floa
     if (v_out && !aligned(v_out, 4)) return fail(DENDSN_ERR_MISALIGNED, "v_out misaligned");
     if (saved && !aligned(saved, 16)) return fail(DENDSN_ERR_MISALIGNED, "saved must be 16-byte aligned");
     FwdArgs a;
-    a.g = pl.g;
+    a.g = pl.gf;
     a.p = make_params(*cfg, alpha, xi, zeta, kappa, mask);
     a.x = x;
     a.spikes = spikes;
     a.v_out = v_out;
-    a.ck_vd = (saved && pl.g.n_ck > 0) ? static_cast<float *>(saved) : nullptr;
+    a.ck_vd = (saved && pl.gf.n_ck > 0) ? static_cast<float *>(saved) : nullptr;
     a.ck_vs = a.ck_vd ? reinterpret_cast<float *>(static_cast<char *>(saved) + pl.ck_vd_bytes)
                       : nullptr;
-    cudaError_t e = dispatch_forward(*cfg, a, pl.blocks, static_cast<cudaStream_t>(stream));
+    cudaError_t e = dispatch_forward(*cfg, a, pl.blocks_f, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess)
         return fail(DENDSN_ERR_CUDA, "forward launch failed: %s", cudaGetErrorString(e));
     g_launches.fetch_add(1, std::memory_order_relaxed);
@@ -287,7 +301,7 @@ dendsn_status dendsn_backward(const dendsn_config *cfg, const void *x, const flo
     if (!aligned(grad_alpha, 4) || !aligned(grad_xi, 4) || !aligned(grad_zeta, 4) ||
         !aligned(grad_kappa, 4))
         return fail(DENDSN_ERR_MISALIGNED, "parameter gradients must be 4-byte aligned");
-    const bool work = pl.g.BN > 0 && pl.g.T > 0;
+    const bool work = pl.gb.BN > 0 && pl.gb.T > 0;
     if (work) {
         if (!x || !grad_spikes || !grad_x)
             return fail(DENDSN_ERR_INVALID_ARG, "x, grad_spikes or grad_x is NULL");
@@ -296,8 +310,8 @@ dendsn_status dendsn_backward(const dendsn_config *cfg, const void *x, const flo
             return fail(DENDSN_ERR_MISALIGNED, "x and grad_x must be 16-byte aligned");
         if (!aligned(grad_spikes, pl.sx)) return fail(DENDSN_ERR_MISALIGNED, "grad_spikes misaligned");
         if (grad_v && !aligned(grad_v, 4)) return fail(DENDSN_ERR_MISALIGNED, "grad_v misaligned");
-        if (pl.g.n_ck > 0 && !saved)
-            return fail(DENDSN_ERR_INVALID_ARG, "T=%d needs the forward's saved checkpoints", pl.g.T);
+        if (pl.gb.n_ck > 0 && !saved)
+            return fail(DENDSN_ERR_INVALID_ARG, "T=%d needs the forward's saved checkpoints", pl.gb.T);
         if (saved && !aligned(saved, 16)) return fail(DENDSN_ERR_MISALIGNED, "saved must be 16-byte aligned");
         if (!scratch) return fail(DENDSN_ERR_INVALID_ARG, "scratch is NULL");
         if (!aligned(scratch, 16)) return fail(DENDSN_ERR_MISALIGNED, "scratch must be 16-byte aligned");
@@ -305,24 +319,24 @@ dendsn_status dendsn_backward(const dendsn_config *cfg, const void *x, const flo
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (work) {
         BwdArgs a;
-        a.g = pl.g;
+        a.g = pl.gb;
         a.p = make_params(*cfg, alpha, xi, zeta, kappa, mask);
         a.x = x;
         a.gs = grad_spikes;
         a.gv = grad_v;
-        a.ck_vd = pl.g.n_ck > 0 ? static_cast<const float *>(saved) : nullptr;
-        a.ck_vs = pl.g.n_ck > 0 ? reinterpret_cast<const float *>(
+        a.ck_vd = pl.gb.n_ck > 0 ? static_cast<const float *>(saved) : nullptr;
+        a.ck_vs = pl.gb.n_ck > 0 ? reinterpret_cast<const float *>(
                                       static_cast<const char *>(saved) + pl.ck_vd_bytes)
                                 : nullptr;
         a.gx = grad_x;
         a.partials = static_cast<float *>(scratch);
-        cudaError_t e = dispatch_backward(*cfg, pl.g.L, a, pl.blocks, s);
+        cudaError_t e = dispatch_backward(*cfg, pl.gb.L, a, pl.blocks_b, s);
         if (e != cudaSuccess)
             return fail(DENDSN_ERR_CUDA, "backward launch failed: %s", cudaGetErrorString(e));
         g_launches.fetch_add(1, std::memory_order_relaxed);
     }
     FinArgs f;
-    f.g = pl.g;
+    f.g = pl.gb;
     f.partials = static_cast<const float *>(scratch);
     f.g_alpha = grad_alpha;
     f.g_xi = grad_xi;

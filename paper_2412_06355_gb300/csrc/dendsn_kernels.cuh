@@ -66,6 +66,33 @@ template <int KT> struct Vec<float, KT> {
     }
 };
 
+// Eight fp32 compartments of one lane: two 16-byte halves.
+struct F8 { float4 a, b; };
+template <> struct Vec<float, 8> {
+    using Raw = F8;
+    static __device__ __forceinline__ Raw load(const float *p) {
+        F8 r;
+        r.a = __ldcs(reinterpret_cast<const float4 *>(p));
+        r.b = __ldcs(reinterpret_cast<const float4 *>(p) + 1);
+        return r;
+    }
+    static __device__ __forceinline__ void unpack(const Raw &r, float (&v)[8]) {
+        v[0] = r.a.x; v[1] = r.a.y; v[2] = r.a.z; v[3] = r.a.w;
+        v[4] = r.b.x; v[5] = r.b.y; v[6] = r.b.z; v[7] = r.b.w;
+    }
+    static __device__ __forceinline__ Raw pack(const float (&v)[8]) {
+        F8 r;
+        r.a = make_float4(v[0], v[1], v[2], v[3]);
+        r.b = make_float4(v[4], v[5], v[6], v[7]);
+        return r;
+    }
+    static __device__ __forceinline__ void store(float *p, const float (&v)[8]) {
+        const F8 r = pack(v);
+        __stcs(reinterpret_cast<float4 *>(p), r.a);
+        __stcs(reinterpret_cast<float4 *>(p) + 1, r.b);
+    }
+};
+
 __device__ __forceinline__ float bf16_lo(uint32_t q) { return __uint_as_float(q << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t q) { return __uint_as_float(q & 0xffff0000u); }
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
@@ -75,18 +102,27 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 
 template <int KT> struct Vec<__nv_bfloat16, KT> {
     using T = __nv_bfloat16;
-    using Raw = typename std::conditional<KT == 4, uint2,
-                typename std::conditional<KT == 2, unsigned int, unsigned short>::type>::type;
+    using Raw = typename std::conditional<KT == 8, uint4,
+                typename std::conditional<KT == 4, uint2,
+                typename std::conditional<KT == 2, unsigned int, unsigned short>::type>::type>::type;
     static __device__ __forceinline__ Raw load(const T *p) {
         return __ldcs(reinterpret_cast<const Raw *>(p));
     }
     static __device__ __forceinline__ void unpack(const Raw &r, float (&v)[KT]) {   // exact
-        if constexpr (KT == 4) { v[0] = bf16_lo(r.x); v[1] = bf16_hi(r.x); v[2] = bf16_lo(r.y); v[3] = bf16_hi(r.y); }
+        if constexpr (KT == 8) {
+            v[0] = bf16_lo(r.x); v[1] = bf16_hi(r.x); v[2] = bf16_lo(r.y); v[3] = bf16_hi(r.y);
+            v[4] = bf16_lo(r.z); v[5] = bf16_hi(r.z); v[6] = bf16_lo(r.w); v[7] = bf16_hi(r.w);
+        }
+        else if constexpr (KT == 4) { v[0] = bf16_lo(r.x); v[1] = bf16_hi(r.x); v[2] = bf16_lo(r.y); v[3] = bf16_hi(r.y); }
         else if constexpr (KT == 2) { v[0] = bf16_lo(r); v[1] = bf16_hi(r); }
         else { v[0] = bf16_lo(r); }
     }
     static __device__ __forceinline__ void store(T *p, const float (&v)[KT]) {
-        if constexpr (KT == 4) {
+        if constexpr (KT == 8) {
+            __stcs(reinterpret_cast<uint4 *>(p),
+                   make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
+                              pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7])));
+        } else if constexpr (KT == 4) {
             __stcs(reinterpret_cast<uint2 *>(p), make_uint2(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3])));
         } else if constexpr (KT == 2) {
             __stcs(reinterpret_cast<unsigned int *>(p), pack_bf16x2(v[0], v[1]));
@@ -116,6 +152,8 @@ template <> struct Scalar<__nv_bfloat16> {
     }
 };
 
+template <typename XT> constexpr int xt_code() { return std::is_same<XT, float>::value ? 0 : 1; }
+
 template <int XT> struct XType;
 template <> struct XType<0> { using type = float; };
 template <> struct XType<1> { using type = __nv_bfloat16; };
@@ -123,7 +161,15 @@ template <> struct XType<1> { using type = __nv_bfloat16; };
 // Mask bits of KTb branches of one lane, as 1.0f / 0.0f.
 template <int KTb>
 __device__ __forceinline__ void load_mask(const uint8_t *m, float (&mk)[KTb]) {
-    if constexpr (KTb == 4) {
+    if constexpr (KTb == 8) {
+        const uint32_t q0 = __ldg(reinterpret_cast<const unsigned int *>(m));
+        const uint32_t q1 = __ldg(reinterpret_cast<const unsigned int *>(m) + 1);
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            mk[b] = ((q0 >> (8 * b)) & 0xffu) ? 1.f : 0.f;
+            mk[4 + b] = ((q1 >> (8 * b)) & 0xffu) ? 1.f : 0.f;
+        }
+    } else if constexpr (KTb == 4) {
         const uint32_t q = __ldg(reinterpret_cast<const unsigned int *>(m));
 #pragma unroll
         for (int b = 0; b < 4; ++b) mk[b] = ((q >> (8 * b)) & 0xffu) ? 1.f : 0.f;
@@ -207,7 +253,7 @@ __device__ __forceinline__ void load_neuron_mask(const Params &P, const Geometry
 
 // ================================================================ paired engine, G = 1
 // Compartment i is branch i. u = V^d/zeta - xi/zeta; r = |u|.
-template <int KT, int PSI>
+template <int KT, int PSI, bool TREE>
 struct PairArith {
     static constexpr int N2 = KT / 2;
     static constexpr int KTb = KT;
@@ -248,8 +294,10 @@ struct PairArith {
 #pragma unroll
         for (int m = 0; m < N2; ++m) s.v[m] = make_float2(v[2 * m], v[2 * m + 1]);
     }
-    // Eqs. methods-compartment, -branch-aggregation, -mexican-hat, -soma-input.
-    static __device__ __forceinline__ float step(const LP &lp, St &vd, const float (&x)[KT]) {
+    // The lane's share of Z as one chain over the pairs (used when the forward and the
+    // backward give a neuron the same lanes; see step for the tree order).
+    static __device__ __forceinline__ float step_chain(const LP &lp, St &vd, const float (&x)[KT],
+                                                       bool residual, float inv_k) {
         float2 zp = f2(0.f);
 #pragma unroll
         for (int m = 0; m < N2; ++m) {
@@ -266,7 +314,55 @@ struct PairArith {
             }
             zp = (m == 0) ? fmul2(lp.km[m], y) : ffma2(lp.km[m], y, zp);
         }
-        return __fadd_rn(zp.x, zp.y);
+        float z = __fadd_rn(zp.x, zp.y);
+        if (residual) {
+            float xs = x[0];
+#pragma unroll
+            for (int i = 1; i < KT; ++i) xs = __fadd_rn(xs, x[i]);
+            z = __fmaf_rn(xs, inv_k, z);
+        }
+        return z;
+    }
+    // Eqs. methods-compartment, -branch-aggregation, -mexican-hat, -soma-input, -residual.
+    // The lane's share of Z is summed in a fixed tree: compartments in groups of four
+    // (two pairs, reduced with one paired multiply and one paired FMA, then the two
+    // halves), plus the group's share of the residual, then the groups pairwise. The
+    // cross-lane butterfly continues the same tree, so the result is bit-identical for
+    // any split of a neuron over 1, 2 or 4 lanes.
+    static __device__ __forceinline__ float step(const LP &lp, St &vd, const float (&x)[KT],
+                                                 bool residual, float inv_k) {
+        if constexpr (!TREE) return step_chain(lp, vd, x, residual, inv_k);
+        constexpr int NG = (N2 + 1) / 2;                          // groups of two pairs
+        float gv[NG];
+#pragma unroll
+        for (int q = 0; q < NG; ++q) {
+            float2 acc = f2(0.f);
+#pragma unroll
+            for (int h = 0; h < 2 && 2 * q + h < N2; ++h) {
+                const int m = 2 * q + h;
+                vd.v[m] = ffma2(lp.a[m], vd.v[m], make_float2(x[2 * m], x[2 * m + 1]));
+                const float2 u = ffma2(vd.v[m], lp.iz[m], lp.nxi[m]);
+                float2 y;
+                if constexpr (PSI == PSI_MEXHAT) {
+                    const float2 ss = fmul2(u, u);
+                    const float2 t = fmul2(f2(kNegHalfLog2e), ss);
+                    const float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
+                    y = ffma2(neg2(ss), e, e);                   // (1 - r^2) e^{-r^2/2}
+                } else {
+                    y = make_float2(fabsf(u.x), fabsf(u.y));     // r
+                }
+                acc = (h == 0) ? fmul2(lp.km[m], y) : ffma2(lp.km[m], y, acc);
+            }
+            gv[q] = __fadd_rn(acc.x, acc.y);
+            if (residual) {
+                float xs = x[4 * q];
+#pragma unroll
+                for (int i = 1; i < 4 && 4 * q + i < KT; ++i) xs = __fadd_rn(xs, x[4 * q + i]);
+                gv[q] = __fmaf_rn(xs, inv_k, gv[q]);
+            }
+        }
+        if constexpr (NG == 2) gv[0] = __fadd_rn(gv[0], gv[NG - 1]);
+        return gv[0];
     }
     static __device__ __forceinline__ void acc_zero(Acc &c) {
 #pragma unroll
@@ -351,7 +447,8 @@ struct ScalarArith {
         return __fmaf_rn(vd, lp.iz[i / G], lp.nxi[i]);
     }
     // Eqs. methods-compartment, -branch-aggregation, -mexican-hat, -soma-input.
-    static __device__ __forceinline__ float step(const LP &lp, St &vd, const float (&x)[KT]) {
+    static __device__ __forceinline__ float step(const LP &lp, St &vd, const float (&x)[KT],
+                                                 bool residual, float inv_k) {
 #pragma unroll
         for (int i = 0; i < KT; ++i) vd.v[i] = __fmaf_rn(lp.a[i], vd.v[i], x[i]);
         float zp = 0.f;
@@ -372,6 +469,12 @@ struct ScalarArith {
                 y = (G == 1) ? fabsf(u0) : sqrtf(ss);         // r
             }
             zp = __fmaf_rn(lp.km[b], y, zp);
+        }
+        if (residual) {
+            float xs = x[0];
+#pragma unroll
+            for (int i = 1; i < KT; ++i) xs = __fadd_rn(xs, x[i]);
+            zp = __fmaf_rn(xs, inv_k, zp);
         }
         return zp;
     }
@@ -446,18 +549,12 @@ struct ScalarArith {
     }
 };
 
-template <int KT, int G, int PSI>
-using Arith = typename std::conditional<(G == 1 && KT % 2 == 0), PairArith<KT, PSI>,
+// fp32 layers sum Z in the group tree (their forward and backward may split a neuron
+// over different lane counts); bf16 layers use the shorter chain.
+template <int KT, int G, int PSI, typename XT>
+using Arith = typename std::conditional<(G == 1 && KT % 2 == 0),
+                                        PairArith<KT, PSI, std::is_same<XT, float>::value>,
                                         ScalarArith<KT, G, PSI>>::type;
-
-// Eq. methods-residual: the lane's share of sum_i X_i (same order in forward and recompute).
-template <int KT>
-__device__ __forceinline__ float lane_input_sum(const float (&x)[KT]) {
-    float xs = x[0];
-#pragma unroll
-    for (int i = 1; i < KT; ++i) xs = __fadd_rn(xs, x[i]);
-    return xs;
-}
 
 // Sum of the LPN lanes' shares (xor butterfly: every lane gets the same bits).
 template <int LPN>
@@ -472,9 +569,7 @@ __device__ __forceinline__ float lanes_sum(float v) {
 template <typename AR, int KT, int LPN>
 __device__ __forceinline__ float soma_input(const typename AR::LP &lp, typename AR::St &vd,
                                             const float (&x)[KT], bool residual, float inv_k) {
-    float zp = AR::step(lp, vd, x);
-    if (residual) zp = __fmaf_rn(lane_input_sum<KT>(x), inv_k, zp);
-    return lanes_sum<LPN>(zp);
+    return lanes_sum<LPN>(AR::step(lp, vd, x, residual, inv_k));
 }
 
 // LIF soma charge with the reset folded in: hard V = beta (1 - S) V + Z
@@ -541,6 +636,16 @@ __device__ __forceinline__ void cp_async(void *smem, const void *gmem, float dep
     else
         asm volatile("cp.async.ca.shared.global [%0], [%1], %3; // %2\n" :: "r"(d), "l"(gmem), "f"(dep), "n"(BYTES) : "memory");
 }
+// Copies one lane's Raw element (4, 8, 16 or 32 bytes) with cp.async.
+template <typename Raw>
+__device__ __forceinline__ void cp_async_raw(Raw *smem, const void *gmem, float dep) {
+    if constexpr (sizeof(Raw) == 32) {
+        cp_async<16>(reinterpret_cast<char *>(smem), gmem, dep);
+        cp_async<16>(reinterpret_cast<char *>(smem) + 16, static_cast<const char *>(gmem) + 16, dep);
+    } else {
+        cp_async<sizeof(Raw)>(smem, gmem, dep);
+    }
+}
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" :: "n"(N) : "memory"); }
@@ -548,13 +653,14 @@ __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_gr
 // x is prefetched kFwdBatch steps ahead of use (a ring of kFwdBatch registers);
 // checkpoints every g.L steps (g.L is a power of two and a multiple of the batch).
 template <int K, int G, int PSI, typename XT>
-__global__ void __launch_bounds__(kThreads, DENDSN_FWD_MINB)
+__global__ void __launch_bounds__(fwd_threads(K), lane_compartments(K) >= 8 ? 2 : DENDSN_FWD_MINB)
 dendsn_forward_kernel(const FwdArgs A) {
-    constexpr int KT = (K < 4) ? K : 4;
+    constexpr int NT = fwd_threads(K);
+    constexpr int KT = lane_compartments(K);
     constexpr int LPN = K / KT;
     constexpr int L = kFwdBatch;
     using V = Vec<XT, KT>;
-    using AR = Arith<KT, G, PSI>;
+    using AR = Arith<KT, G, PSI, XT>;
     constexpr bool ASYNC = DENDSN_FWD_ASYNC && sizeof(typename V::Raw) >= 4;
     const Geometry &g = A.g;
     const Params &P = A.p;
@@ -584,13 +690,13 @@ dendsn_forward_kernel(const FwdArgs A) {
         constexpr int D = kFwdDepth;
         using Raw = typename V::Raw;
         extern __shared__ float4 fwd_smem[];
-        Raw *ring = reinterpret_cast<Raw *>(fwd_smem) + threadIdx.x;     // slot k at ring[k * kThreads]
+        Raw *ring = reinterpret_cast<Raw *>(fwd_smem) + threadIdx.x;     // slot k at ring[k * NT]
         const XT *ip = xrow;                    // next step to fetch
         int it = 0, ir = 0;                     // its step and row
         const int64_t row_jump = rX - (int64_t)T * sX;
 #pragma unroll
         for (int k = 0; k < D; ++k) {
-            if (ir < pos.nrows) cp_async<sizeof(Raw)>(ring + k * kThreads, ip, 0.f);
+            if (ir < pos.nrows) cp_async_raw(ring + k * NT, ip, 0.f);
             cp_async_commit();
             ip += sX;
             if (++it == T) { it = 0; ++ir; ip += row_jump; }
@@ -608,10 +714,10 @@ dendsn_forward_kernel(const FwdArgs A) {
             for (int t = 0; t < T; ++t) {
                 cp_async_wait<D - 1>();
                 float xv[KT];
-                V::unpack(ring[slot * kThreads], xv);
+                V::unpack(ring[slot * NT], xv);
                 const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
                 // the slot's value has been used (z depends on it): refill it
-                if (ir < pos.nrows) cp_async<sizeof(Raw)>(ring + slot * kThreads, ip, z);
+                if (ir < pos.nrows) cp_async_raw(ring + slot * NT, ip, z);
                 cp_async_commit();
                 ip += sX;
                 if (++it == T) { it = 0; ++ir; ip += row_jump; }
@@ -705,23 +811,29 @@ template <int KT, int G>
 constexpr int acc_count() { return 2 * KT + 2 * (KT / G); }
 
 template <int K, int G, int PSI, typename XT, int L>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(bwd_threads(bwd_lane_compartments(K, G, xt_code<XT>(), L)),
+                                  bwd_threads(bwd_lane_compartments(K, G, xt_code<XT>(), L)) == 128 ? 3 : 2)
 dendsn_backward_kernel(const BwdArgs A) {
-    constexpr int KT = (K < 4) ? K : 4;
+    constexpr int KT = bwd_lane_compartments(K, G, xt_code<XT>(), L);
+    constexpr int NT = bwd_threads(KT);
     constexpr int LPN = K / KT;
     constexpr int KTb = KT / G;
     constexpr int NA = acc_count<KT, G>();
     // L == 4 is only used for T <= 4: one chunk per row and never a checkpoint
     constexpr bool MULTI = L > 4;
+    // the recomputed history lives in shared memory for multi-chunk rows and for
+    // 8-compartment lanes (registers), else in registers
+    constexpr bool SHIST = MULTI || KT >= 8;
     constexpr int H = 4;                         // prefetch distance of x in steps
     using V = Vec<XT, KT>;
     using S1 = Scalar<XT>;
-    using AR = Arith<KT, G, PSI>;
+    using AR = Arith<KT, G, PSI, XT>;
     using HistRaw = typename Vec<float, KT>::Raw;
     using XRaw = typename V::Raw;
-    // multi-chunk: x staged through a per-thread cp.async ring in shared memory; single
-    // chunk (T <= 4): a register ring, which measured faster there
-    constexpr bool BASYNC = DENDSN_BWD_ASYNC && MULTI && sizeof(XRaw) >= 4;
+    // x staged through a per-thread cp.async ring in shared memory when the history is
+    // there too; otherwise (T <= 4, up to 4 compartments) a register ring, which
+    // measured faster there
+    constexpr bool BASYNC = DENDSN_BWD_ASYNC && SHIST && sizeof(XRaw) >= 4;
     constexpr int D = kBwdDepth;
     const Geometry &g = A.g;
     const Params &P = A.p;
@@ -745,9 +857,9 @@ dendsn_backward_kernel(const BwdArgs A) {
     const bool residual = P.residual != 0;
 
     extern __shared__ float4 smem_f4[];
-    HistRaw *hist = reinterpret_cast<HistRaw *>(smem_f4);                             // [L][kThreads]
-    float *hist_vs = reinterpret_cast<float *>(hist + (MULTI ? L * kThreads : 0));   // [L][kThreads]
-    XRaw *xring = reinterpret_cast<XRaw *>(hist_vs + (MULTI ? L * kThreads : 0)) + threadIdx.x;   // [D][kThreads]
+    HistRaw *hist = reinterpret_cast<HistRaw *>(smem_f4);                             // [L][NT]
+    float *hist_vs = reinterpret_cast<float *>(hist + (SHIST ? L * NT : 0));   // [L][NT]
+    XRaw *xring = reinterpret_cast<XRaw *>(hist_vs + (SHIST ? L * NT : 0)) + threadIdx.x;   // [D][NT]
     // cp.async walker over this thread's sequence: rows, chunks in reverse, steps forward
     const XT *const xbase = xrow;
     int wr = 0, wc = nc - 1, wt = 0;
@@ -767,7 +879,7 @@ dendsn_backward_kernel(const BwdArgs A) {
     if constexpr (BASYNC) {
 #pragma unroll
         for (int k = 0; k < D; ++k) {
-            if (wr < pos.nrows) cp_async<sizeof(XRaw)>(xring + k * kThreads, wp, 0.f);
+            if (wr < pos.nrows) cp_async_raw(xring + k * NT, wp, 0.f);
             cp_async_commit();
             walk();
         }
@@ -836,9 +948,9 @@ dendsn_backward_kernel(const BwdArgs A) {
 
             // recompute the chunk, keeping V^d and V^s of every step (in registers for a
             // single chunk, in shared memory, one slot per thread and step, otherwise)
-            typename AR::St vdh[MULTI ? 1 : L];
-            float vsh[MULTI ? 1 : L];
-            float gsc[MULTI ? 1 : L];     // single chunk: grad_spikes taken during the recompute
+            typename AR::St vdh[SHIST ? 1 : L];
+            float vsh[SHIST ? 1 : L];
+            float gsc[SHIST ? 1 : L];     // register history: grad_spikes taken during the recompute
             {
                 typename AR::St vd = vd0;
                 float v = v0;
@@ -849,8 +961,8 @@ dendsn_backward_kernel(const BwdArgs A) {
                 for (int tt = 0; tt < L; ++tt) {
                     float xv[KT];
                     if constexpr (!BASYNC) V::unpack(xb[BASYNC ? 0 : tt % H], xv);
-                    if constexpr (!MULTI) {
-                        gsc[MULTI ? 0 : tt] = S1::unpack(gsb[tt]);
+                    if constexpr (!SHIST) {
+                        gsc[SHIST ? 0 : tt] = S1::unpack(gsb[tt]);
                         if (tt < nnext) gsb[tt] = S1::load(gsn + (int64_t)tt * BN);
                     }
                     if constexpr (!BASYNC) {
@@ -867,26 +979,26 @@ dendsn_backward_kernel(const BwdArgs A) {
                     if (tt < ncur) {
                         if constexpr (BASYNC) {
                             cp_async_wait<D - 1>();
-                            V::unpack(xring[xslot * kThreads], xv);
+                            V::unpack(xring[xslot * NT], xv);
                         }
                         const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
                         if constexpr (BASYNC) {
                             // the slot's value has been used (z depends on it): refill it
-                            if (wr < pos.nrows) cp_async<sizeof(XRaw)>(xring + xslot * kThreads, wp, z);
+                            if (wr < pos.nrows) cp_async_raw(xring + xslot * NT, wp, z);
                             cp_async_commit();
                             walk();
                             xslot = (xslot == D - 1) ? 0 : xslot + 1;
                         }
                         v = soma_charge(z, v, s, P);
                         s = v >= P.theta;
-                        if constexpr (MULTI) {
+                        if constexpr (SHIST) {
                             float vda[KT];
                             AR::to_array(vd, vda);
-                            hist[tt * kThreads + threadIdx.x] = Vec<float, KT>::pack(vda);
-                            hist_vs[tt * kThreads + threadIdx.x] = v;
+                            hist[tt * NT + threadIdx.x] = Vec<float, KT>::pack(vda);
+                            hist_vs[tt * NT + threadIdx.x] = v;
                         } else {
-                            vdh[MULTI ? 0 : tt] = vd;
-                            vsh[MULTI ? 0 : tt] = v;
+                            vdh[SHIST ? 0 : tt] = vd;
+                            vsh[SHIST ? 0 : tt] = v;
                         }
                     }
                 }
@@ -897,31 +1009,31 @@ dendsn_backward_kernel(const BwdArgs A) {
 #pragma unroll
             for (int tt = L - 1; tt >= 0; --tt) {
                 float gs_t;
-                if constexpr (MULTI) {
+                if constexpr (SHIST) {
                     gs_t = S1::unpack(gsb[tt]);
                     // refill slot tt with the next chunk's grad_spikes once this one is taken
                     if (tt < nnext) gsb[tt] = S1::load(gsn + (int64_t)tt * BN);
                 } else {
-                    gs_t = gsc[MULTI ? 0 : tt];
+                    gs_t = gsc[SHIST ? 0 : tt];
                 }
                 if (tt < ncur) {
                     float vs;
                     typename AR::St vdt, vdp;                       // V^d[t], V^d[t-1]
-                    if constexpr (MULTI) {
-                        vs = hist_vs[tt * kThreads + threadIdx.x];
+                    if constexpr (SHIST) {
+                        vs = hist_vs[tt * NT + threadIdx.x];
                         float a[KT];
-                        Vec<float, KT>::unpack(hist[tt * kThreads + threadIdx.x], a);
+                        Vec<float, KT>::unpack(hist[tt * NT + threadIdx.x], a);
                         AR::from_array(vdt, a);
                         if (tt > 0) {
-                            Vec<float, KT>::unpack(hist[(tt > 0 ? tt - 1 : 0) * kThreads + threadIdx.x], a);
+                            Vec<float, KT>::unpack(hist[(tt > 0 ? tt - 1 : 0) * NT + threadIdx.x], a);
                             AR::from_array(vdp, a);
                         } else {
                             vdp = vd0;
                         }
                     } else {
-                        vs = vsh[MULTI ? 0 : tt];
-                        vdt = vdh[MULTI ? 0 : tt];
-                        vdp = (tt > 0) ? vdh[MULTI ? 0 : (tt > 0 ? tt - 1 : 0)] : vd0;
+                        vs = vsh[SHIST ? 0 : tt];
+                        vdt = vdh[SHIST ? 0 : tt];
+                        vdp = (tt > 0) ? vdh[SHIST ? 0 : (tt > 0 ? tt - 1 : 0)] : vd0;
                     }
                     const bool st = vs >= P.theta;
                     const float dvds = P.detach ? 0.f : (P.soft ? soft_dvds : __fmul_rn(hard_dvds, vs));
@@ -963,7 +1075,7 @@ dendsn_backward_kernel(const BwdArgs A) {
     if constexpr (BASYNC) cp_async_wait<0>();
     __syncthreads();
 #pragma unroll
-    for (int a = 0; a < NA; ++a) red[a * kThreads + threadIdx.x] = v[a];
+    for (int a = 0; a < NA; ++a) red[a * NT + threadIdx.x] = v[a];
     __syncthreads();
     const int ct = blockIdx.x % g.nCT;
     const int p0 = ct * g.TXn;
@@ -973,7 +1085,7 @@ dendsn_backward_kernel(const BwdArgs A) {
     const int NP = 2 * g.K + 2 * g.Kb;              // per-channel gradient vector
     float *out = A.partials + (int64_t)blockIdx.x * g.nch_max * NP;
     const int items = nch * LPN * NA;
-    for (int w = threadIdx.x; w < items; w += kThreads) {
+    for (int w = threadIdx.x; w < items; w += NT) {
         const int a = w % NA;
         const int sub = (w / NA) % LPN;
         const int lc = w / (NA * LPN);
@@ -983,7 +1095,7 @@ dendsn_backward_kernel(const BwdArgs A) {
         float sum = 0.f;
         for (int ry = 0; ry < g.TY; ++ry)
             for (int cx = cx_lo; cx < cx_hi; cx += g.seg)
-                sum = __fadd_rn(sum, red[a * kThreads + (ry * g.TXn + cx) * LPN + sub]);
+                sum = __fadd_rn(sum, red[a * NT + (ry * g.TXn + cx) * LPN + sub]);
         int slot;
         if (a < KT) slot = sub * KT + a;                                        // alpha
         else if (a < 2 * KT) slot = g.K + sub * KT + (a - KT);                  // xi
@@ -1004,27 +1116,30 @@ cudaError_t allow_smem(Kern kernel, size_t bytes) {
 template <int K, int G, int PSI, int XT>
 cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s) {
     using T = typename XType<XT>::type;
-    constexpr int KT = (K < 4) ? K : 4;
+    constexpr int KT = lane_compartments(K);
     constexpr size_t raw = sizeof(typename Vec<T, KT>::Raw);
-    const size_t smem = (DENDSN_FWD_ASYNC && raw >= 4) ? raw * kFwdDepth * kThreads : 0;
+    constexpr int NT = fwd_threads(K);
+    const size_t smem = (DENDSN_FWD_ASYNC && raw >= 4) ? raw * kFwdDepth * NT : 0;
     cudaError_t e = allow_smem(dendsn_forward_kernel<K, G, PSI, T>, smem);
     if (e != cudaSuccess) return e;
-    dendsn_forward_kernel<K, G, PSI, T><<<blocks, kThreads, smem, s>>>(a);
+    dendsn_forward_kernel<K, G, PSI, T><<<blocks, NT, smem, s>>>(a);
     return cudaGetLastError();
 }
 
 template <int K, int G, int PSI, int XT, int L>
 cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
     using T = typename XType<XT>::type;
-    constexpr int KT = (K < 4) ? K : 4;
-    const size_t red = sizeof(float) * acc_count<KT, G>() * kThreads;
-    const size_t hist = (L > 4) ? sizeof(float) * (KT + 1) * L * kThreads : 0;
+    constexpr int KT = bwd_lane_compartments(K, G, XT, L);
+    constexpr int NT = bwd_threads(KT);
+    const size_t red = sizeof(float) * acc_count<KT, G>() * NT;
+    constexpr bool shist = (L > 4) || KT >= 8;
+    const size_t hist = shist ? sizeof(float) * (KT + 1) * L * NT : 0;
     constexpr size_t xraw = sizeof(typename Vec<T, KT>::Raw);
-    const size_t ring = (DENDSN_BWD_ASYNC && L > 4 && xraw >= 4) ? xraw * kBwdDepth * kThreads : 0;
+    const size_t ring = (DENDSN_BWD_ASYNC && shist && xraw >= 4) ? xraw * kBwdDepth * NT : 0;
     const size_t smem = red > hist + ring ? red : hist + ring;
     cudaError_t e = allow_smem(dendsn_backward_kernel<K, G, PSI, T, L>, smem);
     if (e != cudaSuccess) return e;
-    dendsn_backward_kernel<K, G, PSI, T, L><<<blocks, kThreads, smem, s>>>(a);
+    dendsn_backward_kernel<K, G, PSI, T, L><<<blocks, NT, smem, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -8,8 +8,21 @@ namespace dendsn {
 
 enum { PSI_IDENTITY = 0, PSI_MEXHAT = 1 };
 
-constexpr int kThreads = 256;     // threads per block of the forward/backward kernels
 constexpr int kFwdBatch = 4;      // time steps per load batch in the forward
+
+// Compartments one lane owns in the forward (a neuron is served by K / that many lanes).
+constexpr int lane_compartments(int K) { return K < 8 ? K : 8; }
+// In the backward, 8 fp32 compartments per lane with T <= 4 measured slower than two
+// lanes of 4 (their registers force the history into shared memory for a very short
+// sequence), so that case splits. fp32 layers sum Z in an order that is the same for
+// both splits (the paired engine's group tree).
+constexpr int bwd_lane_compartments(int K, int G, int xt, int L) {
+    return (K >= 8 && G == 1 && xt == 0 && L <= 4) ? 4 : lane_compartments(K);
+}
+// Threads per block: the forward always 256; the backward 128 when a lane owns 8
+// compartments (its ~165 registers allow three 128-thread blocks per SM).
+constexpr int fwd_threads(int K) { return 256; }
+constexpr int bwd_threads(int KT) { return KT >= 8 ? 128 : 256; }
 
 // Tiling and sizes shared by every kernel of one call (computed on the host).
 // Neuron j = o * P + p: row o in [0, O), column p in [0, P); channel = p / inner.

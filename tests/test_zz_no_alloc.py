@@ -65,9 +65,9 @@ def test_noalloc_backward_matches_backward_twice_in_a_row():
 def test_noalloc_rejects_layers_beyond_its_buffer():
     if not torch.cuda.is_available():
         pytest.fail("needs a CUDA device")
-    # 65536 channels of one neuron each: every block touches 33 channels, and the
-    # per-block partials need 8.25 MiB, just over the built-in 8 MiB
-    w = workloads.Workload("huge", T=1, B=32, N=65536, K=4, G=1, C=65536, inner=1,
+    # 65536 channels of one neuron each with 16 compartments: every block keeps
+    # partials for all the channels of its columns, 16 MiB in all, twice the built-in 8 MiB
+    w = workloads.Workload("huge", T=1, B=32, N=65536, K=16, G=1, C=65536, inner=1,
                            dtype="f32", psi="mh", reset="hard")
     cfg = binding.config_of(w)
     _, need = binding.dendsn_workspace_size(cfg)
@@ -75,4 +75,4 @@ def test_noalloc_rejects_layers_beyond_its_buffer():
     d = torch.empty(16, device="cuda")
     with pytest.raises(binding.DendSNError) as e:
         binding.dendsn_backward_noalloc(cfg, d, d, d, d, d, None, d, None, None, d, d, d, d, d)
-    assert e.value.status == 2 and "8388608" in str(e.value)
+    assert e.value.status == 2 and "8388608" in str(e.value) and str(need) in str(e.value)
