@@ -701,46 +701,80 @@ dendsn_forward_kernel(const FwdArgs A) {
             ip += sX;
             if (++it == T) { it = 0; ++ir; ip += row_jump; }
         }
-        int slot = 0;
-        int64_t j = j0;
-        for (int i = 0; i < pos.nrows; ++i) {
-            if (P.mask_mode == 2) AR::neuron_mask(P, g, j % g.N, pos.chan, pos.sub, lp);
-            typename AR::St vd;
-            AR::zero(vd);
-            float v = 0.f;
-            bool s = false;
-            XT *sp = srow;
-            float *vp = vrow;
-            for (int t = 0; t < T; ++t) {
-                cp_async_wait<D - 1>();
-                float xv[KT];
-                V::unpack(ring[slot * NT], xv);
-                const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
-                // the slot's value has been used (z depends on it): refill it
-                if (ir < pos.nrows) cp_async_raw(ring + slot * NT, ip, z);
-                cp_async_commit();
-                ip += sX;
-                if (++it == T) { it = 0; ++ir; ip += row_jump; }
-                v = soma_charge(z, v, s, P);
-                s = v >= P.theta;                          // Eq. methods-lif-fire
-                if (store) {
-                    Scalar<XT>::store_spike(sp, s);
-                    if (vp) __stcs(vp, v);
+        // The step loop is specialised on whether V^s and checkpoints are written and on
+        // whether T divides the ring depth (then the step fetched D steps ahead is the
+        // same step D/T rows further on: no walker needed).
+        auto rows = [&](auto extra, auto div) {
+            // EXTRA: V^s output and/or checkpoints requested (each still tested inside)
+            constexpr bool EXTRA = decltype(extra)::value, DIV = decltype(div)::value;
+            int slot = 0;
+            int64_t j = j0;
+            const int rows_ahead = DIV ? D / T : 0;
+            const int64_t ahead = (int64_t)rows_ahead * rX;
+            const XT *xr = xrow;
+            XT *sr = srow;
+            float *vr = vrow;
+            for (int i = 0; i < pos.nrows; ++i) {
+                if (P.mask_mode == 2) AR::neuron_mask(P, g, j % g.N, pos.chan, pos.sub, lp);
+                typename AR::St vd;
+                AR::zero(vd);
+                float v = 0.f;
+                bool s = false;
+                XT *sp = sr;
+                float *vp = vr;
+                const XT *cp = xr;                       // this step's x in global memory
+                const bool fetch_row = i + rows_ahead < pos.nrows;
+                for (int t = 0; t < T; ++t) {
+                    cp_async_wait<D - 1>();
+                    float xv[KT];
+                    V::unpack(ring[slot * NT], xv);
+                    const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
+                    // the slot's value has been used (z depends on it): refill it
+                    if constexpr (DIV) {
+                        if (fetch_row) cp_async_raw(ring + slot * NT, cp + ahead, z);
+                        cp += sX;
+                    } else {
+                        if (ir < pos.nrows) cp_async_raw(ring + slot * NT, ip, z);
+                        ip += sX;
+                        if (++it == T) { it = 0; ++ir; ip += row_jump; }
+                    }
+                    cp_async_commit();
+                    v = soma_charge(z, v, s, P);
+                    s = v >= P.theta;                      // Eq. methods-lif-fire
+                    if (store) {
+                        Scalar<XT>::store_spike(sp, s);
+                        if constexpr (EXTRA) {
+                            if (vp) __stcs(vp, v);
+                        }
+                    }
+                    sp += BN;
+                    if constexpr (EXTRA) {
+                        if (vp) vp += BN;
+                        if (write_ck && ((t + 1) & (g.L - 1)) == 0 && t + 1 < T) {
+                            const int ck = (t + 1) / g.L - 1;
+                            float vda[KT];
+                            AR::to_array(vd, vda);
+                            Vec<float, KT>::store(A.ck_vd + ((int64_t)ck * BN + j) * K + pos.sub * KT, vda);
+                            if (pos.sub == 0) __stcs(A.ck_vs + (int64_t)ck * BN + j, v);
+                        }
+                    }
+                    slot = (slot == D - 1) ? 0 : slot + 1;
                 }
-                sp += BN;
-                if (vp) vp += BN;
-                if (write_ck && ((t + 1) & (g.L - 1)) == 0 && t + 1 < T) {
-                    const int ck = (t + 1) / g.L - 1;
-                    float vda[KT];
-                    AR::to_array(vd, vda);
-                    Vec<float, KT>::store(A.ck_vd + ((int64_t)ck * BN + j) * K + pos.sub * KT, vda);
-                    if (pos.sub == 0) __stcs(A.ck_vs + (int64_t)ck * BN + j, v);
+                xr += rX;
+                sr += jstep;
+                if constexpr (EXTRA) {
+                    if (vr) vr += jstep;
                 }
-                slot = (slot == D - 1) ? 0 : slot + 1;
+                j += jstep;
             }
-            srow += jstep;
-            if (vrow) vrow += jstep;
-            j += jstep;
+        };
+        using yes = std::true_type;
+        using no = std::false_type;
+        const bool div = (D % T) == 0;
+        if (vrow != nullptr || write_ck) {
+            if (div) rows(yes{}, yes{}); else rows(yes{}, no{});
+        } else {
+            if (div) rows(no{}, yes{}); else rows(no{}, no{});
         }
         cp_async_wait<0>();
         return;
@@ -852,9 +886,13 @@ dendsn_backward_kernel(const BwdArgs A) {
     const XT *__restrict__ gsrow = static_cast<const XT *>(A.gs) + j0;
     XT *__restrict__ gxrow = static_cast<XT *>(A.gx) + j0 * K + pos.sub * KT;
     const float *gvrow = A.gv ? A.gv + j0 : nullptr;
-    const float hard_dvds = -P.beta;             // dV[t+1]/dS[t] = -beta V[t]
-    const float soft_dvds = -P.beta * P.theta;   // dV[t+1]/dS[t] = -beta theta
+    // dV[t+1]/dS[t] = kv V[t] + cs: hard -beta V[t], soft -beta theta, 0 when detached;
+    // dV[t+1]/dV[t] = beta, or b_spike after a spike (0 hard, beta soft)
+    const float kv = (P.detach || P.soft) ? 0.f : -P.beta;
+    const float cs = (P.detach || !P.soft) ? 0.f : -P.beta * P.theta;
+    const float b_spike = P.soft ? P.beta : 0.f;
     const bool residual = P.residual != 0;
+    const bool has_gv = A.gv != nullptr;
 
     extern __shared__ float4 smem_f4[];
     HistRaw *hist = reinterpret_cast<HistRaw *>(smem_f4);                             // [L][NT]
@@ -957,13 +995,15 @@ dendsn_backward_kernel(const BwdArgs A) {
                 bool s = (!MULTI || c == 0) ? false : (v0 >= P.theta);
                 const XT *xa = xrow + (int64_t)(t0 + H) * sX;      // this chunk, H steps ahead
                 const XT *xnn = xn;                                 // next chunk, from its start
+                const XT *gq = gsn;                                 // next chunk's grad_spikes
 #pragma unroll
                 for (int tt = 0; tt < L; ++tt) {
                     float xv[KT];
                     if constexpr (!BASYNC) V::unpack(xb[BASYNC ? 0 : tt % H], xv);
                     if constexpr (!SHIST) {
                         gsc[SHIST ? 0 : tt] = S1::unpack(gsb[tt]);
-                        if (tt < nnext) gsb[tt] = S1::load(gsn + (int64_t)tt * BN);
+                        if (tt < nnext) gsb[tt] = S1::load(gq);
+                        gq += BN;
                     }
                     if constexpr (!BASYNC) {
                         // refill the slot with the step H ahead: later in this chunk, or
@@ -1005,14 +1045,16 @@ dendsn_backward_kernel(const BwdArgs A) {
             }
             // reverse-time recursion over the chunk
             XT *gxp = gxrow + (int64_t)(t0 + L - 1) * sX;
-            const float *gvp = gvrow ? gvrow + (int64_t)(t0 + L - 1) * BN : nullptr;
+            const float *gvp = has_gv ? gvrow + (int64_t)(t0 + L - 1) * BN : nullptr;
+            const XT *gqr = gsn + (int64_t)(L - 1) * BN;            // next chunk's grad_spikes
 #pragma unroll
             for (int tt = L - 1; tt >= 0; --tt) {
                 float gs_t;
                 if constexpr (SHIST) {
                     gs_t = S1::unpack(gsb[tt]);
                     // refill slot tt with the next chunk's grad_spikes once this one is taken
-                    if (tt < nnext) gsb[tt] = S1::load(gsn + (int64_t)tt * BN);
+                    if (tt < nnext) gsb[tt] = S1::load(gqr);
+                    gqr -= BN;
                 } else {
                     gs_t = gsc[SHIST ? 0 : tt];
                 }
@@ -1036,25 +1078,25 @@ dendsn_backward_kernel(const BwdArgs A) {
                         vdp = (tt > 0) ? vdh[SHIST ? 0 : (tt > 0 ? tt - 1 : 0)] : vd0;
                     }
                     const bool st = vs >= P.theta;
-                    const float dvds = P.detach ? 0.f : (P.soft ? soft_dvds : __fmul_rn(hard_dvds, vs));
-                    const float dvdv = (P.soft || !st) ? P.beta : 0.f;   // beta (1 - S[t]) when hard
+                    const float dvds = __fmaf_rn(kv, vs, cs);               // dV[t+1]/dS[t]
+                    const float dvdv = st ? b_spike : P.beta;               // dV[t+1]/dV[t]
                     const float ds = __fmaf_rn(dvds, dvn, gs_t);                          // dL/dS[t]
                     float dv = __fmaf_rn(surrogate(__fsub_rn(vs, P.theta)), ds,
                                          __fmul_rn(dvdv, dvn));                          // dL/dV^s[t]
-                    if (gvp) dv = __fadd_rn(dv, __ldcs(gvp));
+                    if (has_gv) dv = __fadd_rn(dv, __ldcs(gvp));
                     float gxv[KT];
                     AR::backward(lp, vdt, vdp, dv, Ad, acc, residual ? __fmul_rn(dv, inv_k) : 0.f, gxv);
                     if (pos.active) V::store(gxp, gxv);
                     dvn = dv;
                 }
                 gxp -= sX;
-                if (gvp) gvp -= BN;
+                if (has_gv) gvp -= BN;
             }
         }
         xrow += rX;
         gsrow += jstep;
         gxrow += rX;
-        if (gvrow) gvrow += jstep;
+        if (has_gv) gvrow += jstep;
         j += jstep;
     }
 

@@ -78,7 +78,19 @@ def run_gpu(w, inp_dev: dict, gs, gv, want_v=True):
                            saved=saved)
     g = binding.backward(cfg, inp_dev["x"], inp_dev["alpha"], inp_dev["xi"], inp_dev["zeta"],
                          inp_dev["kappa"], inp_dev["mask"], gs, gv, saved, scratch)
+    # the production forward (no V^s output; checkpoints when T needs them) must give
+    # the same spikes and the same checkpoints bit for bit
+    saved2, _ = binding.workspace(cfg)
+    s2, _ = binding.forward(cfg, inp_dev["x"], inp_dev["alpha"], inp_dev["xi"], inp_dev["zeta"],
+                            inp_dev["kappa"], inp_dev["mask"], want_v=False, saved=saved2)
     torch.cuda.synchronize()
+    assert torch.equal(s, s2), "forward without V^s output changed the spikes"
+    if saved is not None:
+        # checkpoints: (ceil(T/8) - 1) x B*N x (K + 1) float32; the rest is alignment padding
+        n_ck = (w.T + 7) // 8 - 1
+        used = n_ck * w.B * w.N * (w.K + 1) * 4
+        assert torch.equal(saved[:used], saved2[:used]), \
+            "forward without V^s output changed the checkpoints"
     out = {"s": oracle.to_f64(s), "v": None if v is None else oracle.to_f64(v)}
     out.update({k: oracle.to_f64(t) for k, t in g.items()})
     return out
