@@ -46,6 +46,8 @@ def parse_args():
     ap.add_argument("--psi", choices=["mh", "identity"], default=None)
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch B (smaller profiling captures)")
+    ap.add_argument("--variant", choices=["stateful", "stateless", "resstateless", "resstateful"],
+                    default="stateful", help="dendrite variant (Methods, DendSN variants)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU time of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -211,6 +213,9 @@ def workload_of(args):
         w = w.with_(psi=args.psi)
     if args.batch:
         w = w.with_(B=args.batch)
+    if args.variant != "stateful":
+        w = w.with_(stateless=args.variant in ("stateless", "resstateless"),
+                    residual=args.variant.startswith("res"))
     return w
 
 
@@ -219,7 +224,8 @@ def config_dict(w, extra=None):
          "inner": w.inner, "x_dtype": w.dtype, "psi": w.psi, "reset": w.reset,
          "mask": (None if w.mask_p is None else
                   f"Bernoulli({w.mask_p}) per {'neuron' if w.mask_per_neuron else 'channel'}"),
-         "x_density": w.x_density}
+         "x_density": w.x_density,
+         "variant": ("res" if w.residual else "") + ("stateless" if w.stateless else "stateful")}
     if extra:
         d.update(extra)
     return d

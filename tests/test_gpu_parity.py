@@ -184,9 +184,16 @@ def sample_neurons(w, count, seed):
     return flat // w.N, flat % w.N
 
 
-@pytest.mark.parametrize("name", list(WORKLOADS))
-def test_full_size_sampled(name):
-    w = WORKLOADS[name]
+FULL = [(n, {}) for n in WORKLOADS] + [
+    ("conv", dict(stateless=True, residual=True)),        # ResStateless (the Tiny ImageNet choice)
+    ("conv", dict(stateless=True)),                       # Stateless (the CIFAR10-DVS choice)
+    ("event", dict(residual=True, psi="identity")),       # ResStateful, identity branches
+]
+
+
+@pytest.mark.parametrize("name,kw", FULL, ids=[n + "".join(f"-{k}" for k in kw) for n, kw in FULL])
+def test_full_size_sampled(name, kw):
+    w = WORKLOADS[name].with_(**kw)
     cfg = binding.config_of(w)
     inp = workloads.make_inputs(w, "cuda")          # full size, generated on the device
     b_idx, n_idx = sample_neurons(w, 3000, seed=w.seed)
@@ -197,7 +204,8 @@ def test_full_size_sampled(name):
     chan = ((n_idx // w.inner) % w.C).astype(np.int32)
     mrow = (n_idx if w.mask_per_neuron else chan).astype(np.int32)
     ocfg = oracle.OracleConfig(T=w.T, K=w.K, G=w.G, C=w.C, psi=w.psi, reset=w.reset,
-                               theta=w.theta, beta=w.beta)
+                               theta=w.theta, beta=w.beta, stateless=w.stateless,
+                               residual=w.residual)
     prm = [inp[k].cpu() for k in ("alpha", "xi", "zeta", "kappa")]
     mask = None if inp["mask"] is None else inp["mask"].cpu()
     s_o, v_o = oracle.forward(ocfg, xs, chan, mrow, *prm, mask)
