@@ -194,7 +194,11 @@ def cpu_inputs_from(w, inp):
         M = min(M, w.B * w.N)
         flat = torch.arange(M, device=inp["x"].device) * ((w.B * w.N) // M)
         b, n = flat // w.N, flat % w.N
-        x = inp["x"][:, b, n, :].cpu()
+        if w.layout == "paper":                 # [T, B, N/inner, K, inner] -> [T, M, K]
+            x5 = inp["x"].reshape(w.T, w.B, w.N // w.inner, w.K, w.inner)
+            x = x5[:, b, n // w.inner, :, n % w.inner].transpose(0, 1).cpu()
+        else:
+            x = inp["x"][:, b, n, :].cpu()
         gs = inp["gs"][:, b, n].cpu()
         nn = n.cpu().numpy()
         chan = ((nn // w.inner) % w.C).astype(np.int32)
@@ -224,7 +228,7 @@ def config_dict(w, extra=None):
          "inner": w.inner, "x_dtype": w.dtype, "psi": w.psi, "reset": w.reset,
          "mask": (None if w.mask_p is None else
                   f"Bernoulli({w.mask_p}) per {'neuron' if w.mask_per_neuron else 'channel'}"),
-         "x_density": w.x_density,
+         "x_density": w.x_density, "layout": w.layout,
          "variant": ("res" if w.residual else "") + ("stateless" if w.stateless else "stateful")}
     if extra:
         d.update(extra)
@@ -309,7 +313,7 @@ def run_ours(args):
     x, gs = inp["x"], inp["gs"]
     alpha, xi, zeta, kappa, mask = (inp[k] for k in ("alpha", "xi", "zeta", "kappa", "mask"))
     saved, scratch = binding.workspace(cfg, dev)
-    spikes = torch.empty(x.shape[:3], dtype=x.dtype, device=dev)
+    spikes = torch.empty((w.T, w.B, w.N), dtype=x.dtype, device=dev)
     gx = torch.empty_like(x)
     grads, views = distributed.param_grad_buffer(w.C, w.K, w.Kb, dev)
     ga, gxi, gz, gk = (views[k] for k in ("galpha", "gxi", "gzeta", "gkappa"))

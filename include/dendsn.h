@@ -27,7 +27,8 @@
  *    A failed launch returns DENDSN_ERR_CUDA. dendsn_last_error() describes the most
  *    recent failure of the calling thread.
  *  - Layouts are dense row-major:
- *      x, grad_x            [T, B, N, K]   dtype x_dtype; base 16-byte aligned
+ *      x, grad_x            [T, B, N, K] (or the PAPER layout, see dendsn_layout),
+ *                           dtype x_dtype; base 16-byte aligned
  *      spikes, grad_spikes  [T, B, N]      dtype x_dtype (spikes are exactly 0 or 1)
  *      v_out, grad_v        [T, B, N]      float32
  *      alpha, xi            [C, K]         float32
@@ -68,6 +69,15 @@ typedef enum { DENDSN_PSI_IDENTITY = 0, DENDSN_PSI_MEXHAT = 1 } dendsn_psi;
 typedef enum { DENDSN_RESET_HARD = 0, DENDSN_RESET_SOFT = 1 } dendsn_reset;
 /* ATAN: Eq. methods-sg, the only surrogate the paper uses. */
 typedef enum { DENDSN_SG_ATAN = 0 } dendsn_surrogate;
+/*
+ * Layout of x and grad_x (spikes and the other [T, B, N] tensors are the same in both):
+ *   KINNER: [T, B, N, K], a neuron's K compartments contiguous.
+ *   PAPER : [T, B, N / inner, K, inner], i.e. a conv layer's output [T, B, C_o * P, H, W]
+ *           read as (C_o, P, H, W) with inner = H * W (Methods, "Dendritic spiking neural
+ *           networks"): compartment k of neuron n is (n / inner) * K * inner + k * inner
+ *           + n % inner elements into the sample. No transpose is needed.
+ */
+typedef enum { DENDSN_LAYOUT_KINNER = 0, DENDSN_LAYOUT_PAPER = 1 } dendsn_layout;
 
 typedef struct {
     int32_t T, B, N;        /* time steps, samples, neurons per sample */
@@ -83,6 +93,7 @@ typedef struct {
     int32_t mask_per_neuron;/* 0: mask is [C, Kb]; 1: mask is [N, Kb] */
     int32_t stateless;      /* 1: Stateless Dendrite, V^d = X (Methods, "Stateless compartment") */
     int32_t residual;       /* 1: Z += mean_i X_i (Eq. methods-residual) */
+    int32_t layout;         /* dendsn_layout of x and grad_x */
 } dendsn_config;
 
 /*

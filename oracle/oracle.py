@@ -202,10 +202,32 @@ def _cfg_of(w, **over) -> OracleConfig:
     return OracleConfig(**kw)
 
 
+def layer_x(w, x) -> np.ndarray:
+    """A layer's input currents as [T, B*N, K] float64, whatever layout they are stored in.
+
+    "kinner": [T, B, N, K]. "paper": a conv layer's output channels grouped as
+    (C_o, P, H, W) (Methods, "Dendritic spiking neural networks"), i.e.
+    [T, B, N / inner, K, inner] with inner = H*W: compartment k of neuron n sits at
+    [n // inner, k, n % inner].
+    """
+    x = to_f64(x)
+    if getattr(w, "layout", "kinner") == "paper":
+        x = x.reshape(w.T, w.B, w.N // w.inner, w.K, w.inner).transpose(0, 1, 2, 4, 3)
+    return np.ascontiguousarray(x.reshape(w.T, w.B * w.N, w.K))
+
+
+def layer_gx(w, gx: np.ndarray) -> np.ndarray:
+    """[T, B*N, K] -> the layout layer_x reads (gradients share the input's layout)."""
+    if getattr(w, "layout", "kinner") == "paper":
+        gx = gx.reshape(w.T, w.B, w.N // w.inner, w.inner, w.K).transpose(0, 1, 2, 4, 3)
+        return np.ascontiguousarray(gx)
+    return gx.reshape(w.T, w.B, w.N, w.K)
+
+
 def forward_layer(w, inp, **over):
     """Oracle forward of a whole workload `w` with inputs from make_inputs."""
     chan, mrow = layer_channels(w.B, w.N, w.C, w.inner, w.mask_per_neuron)
-    x = to_f64(inp["x"]).reshape(w.T, w.B * w.N, w.K)
+    x = layer_x(w, inp["x"])
     s, v = forward(_cfg_of(w, **over), x, chan, mrow, inp["alpha"], inp["xi"],
                    inp["zeta"], inp["kappa"], inp.get("mask"))
     return s.reshape(w.T, w.B, w.N), v.reshape(w.T, w.B, w.N)
@@ -214,9 +236,9 @@ def forward_layer(w, inp, **over):
 def backward_layer(w, inp, gs=None, **over):
     """Oracle backward of a whole workload `w`; gs overrides inp['gs']."""
     chan, mrow = layer_channels(w.B, w.N, w.C, w.inner, w.mask_per_neuron)
-    x = to_f64(inp["x"]).reshape(w.T, w.B * w.N, w.K)
+    x = layer_x(w, inp["x"])
     gs = inp["gs"] if gs is None else gs
     out = backward(_cfg_of(w, **over), x, chan, mrow, inp["alpha"], inp["xi"], inp["zeta"],
                    inp["kappa"], inp.get("mask"), gs, inp.get("gv"))
-    out["gx"] = out["gx"].reshape(w.T, w.B, w.N, w.K)
+    out["gx"] = layer_gx(w, out["gx"])
     return out

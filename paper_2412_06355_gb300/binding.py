@@ -39,28 +39,33 @@ class dendsn_config(ctypes.Structure):
                 ("surrogate", ctypes.c_int32), ("theta", ctypes.c_float),
                 ("beta", ctypes.c_float), ("detach_reset", ctypes.c_int32),
                 ("mask_per_neuron", ctypes.c_int32), ("stateless", ctypes.c_int32),
-                ("residual", ctypes.c_int32)]
+                ("residual", ctypes.c_int32), ("layout", ctypes.c_int32)]
 
     @property
     def Kb(self) -> int:
         return self.K // self.G
 
 
+LAYOUT_KINNER, LAYOUT_PAPER = 0, 1
+
+
 def make_config(T, B, N, K, G=1, C=1, inner=1, dtype="f32", psi="mh", reset="hard",
                 theta=1.0, beta=0.5, detach_reset=False, mask_per_neuron=False,
-                stateless=False, residual=False, surrogate=SG_ATAN) -> dendsn_config:
+                stateless=False, residual=False, surrogate=SG_ATAN,
+                layout="kinner") -> dendsn_config:
     return dendsn_config(T, B, N, K, G, C, inner, BF16 if dtype == "bf16" else F32,
                          PSI_MEXHAT if psi == "mh" else PSI_IDENTITY,
                          RESET_SOFT if reset == "soft" else RESET_HARD, surrogate,
                          float(theta), float(beta), int(detach_reset), int(mask_per_neuron),
-                         int(stateless), int(residual))
+                         int(stateless), int(residual),
+                         LAYOUT_PAPER if layout == "paper" else LAYOUT_KINNER)
 
 
 def config_of(w) -> dendsn_config:
     """Config of a workloads.Workload."""
     return make_config(w.T, w.B, w.N, w.K, w.G, w.C, w.inner, w.dtype, w.psi, w.reset,
                        w.theta, w.beta, w.detach_reset, w.mask_per_neuron, w.stateless,
-                       w.residual)
+                       w.residual, layout=w.layout)
 
 
 _lib = None
@@ -129,8 +134,35 @@ def dendsn_workspace_size(cfg: dendsn_config):
     return int(s.value), int(w.value)
 
 
+def _need(cfg, **tensors):
+    """Refuses on the host any tensor smaller than what the config makes the kernels touch."""
+    T, B, N, K, C, Kb = cfg.T, cfg.B, cfg.N, cfg.K, cfg.C, cfg.K // cfg.G
+    sx = 2 if cfg.x_dtype == BF16 else 4
+    elems = {"x": T * B * N * K * sx, "grad_x": T * B * N * K * sx,
+             "spikes": T * B * N * sx, "grad_spikes": T * B * N * sx,
+             "v_out": T * B * N * 4, "grad_v": T * B * N * 4,
+             "alpha": C * K * 4, "xi": C * K * 4, "grad_alpha": C * K * 4, "grad_xi": C * K * 4,
+             "zeta": C * Kb * 4, "kappa": C * Kb * 4, "grad_zeta": C * Kb * 4,
+             "grad_kappa": C * Kb * 4, "mask": (N if cfg.mask_per_neuron else C) * Kb}
+    sizes = None
+    for name, t in tensors.items():
+        if t is None:
+            continue
+        if name in ("saved", "scratch"):
+            if sizes is None:
+                sizes = dict(zip(("saved", "scratch"), dendsn_workspace_size(cfg)))
+            need = sizes[name]
+        else:
+            need = elems[name]
+        have = t.numel() * t.element_size()
+        if have < need:
+            raise ValueError(f"{name}: {have} bytes, the config needs {need}")
+
+
 def dendsn_forward(cfg, x, alpha, xi, zeta, kappa, mask, spikes, v_out=None, saved=None,
                    stream=None):
+    _need(cfg, x=x, alpha=alpha, xi=xi, zeta=zeta, kappa=kappa, mask=mask, spikes=spikes,
+          v_out=v_out, saved=saved)
     _check("dendsn_forward", load().dendsn_forward(
         ctypes.byref(cfg), _ptr(x), _ptr(alpha), _ptr(xi), _ptr(zeta), _ptr(kappa),
         _ptr(mask), _ptr(spikes), _ptr(v_out), _ptr(saved), _stream(stream)))
@@ -138,6 +170,10 @@ def dendsn_forward(cfg, x, alpha, xi, zeta, kappa, mask, spikes, v_out=None, sav
 
 def dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved, grad_x,
                     grad_alpha, grad_xi, grad_zeta, grad_kappa, scratch, stream=None):
+    _need(cfg, x=x, alpha=alpha, xi=xi, zeta=zeta, kappa=kappa, mask=mask,
+          grad_spikes=grad_spikes, grad_v=grad_v, saved=saved, grad_x=grad_x,
+          grad_alpha=grad_alpha, grad_xi=grad_xi, grad_zeta=grad_zeta, grad_kappa=grad_kappa,
+          scratch=scratch)
     _check("dendsn_backward", load().dendsn_backward(
         ctypes.byref(cfg), _ptr(x), _ptr(alpha), _ptr(xi), _ptr(zeta), _ptr(kappa),
         _ptr(mask), _ptr(grad_spikes), _ptr(grad_v), _ptr(saved), _ptr(grad_x),
@@ -156,6 +192,9 @@ def dendsn_backward_noalloc(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, g
     for the sharing rules of the built-in buffer.
     """
     global _noalloc_ready
+    _need(cfg, x=x, alpha=alpha, xi=xi, zeta=zeta, kappa=kappa, mask=mask,
+          grad_spikes=grad_spikes, grad_v=grad_v, saved=saved, grad_x=grad_x,
+          grad_alpha=grad_alpha, grad_xi=grad_xi, grad_zeta=grad_zeta, grad_kappa=grad_kappa)
     lib = load()
     if not _noalloc_ready:
         lib.dendsn_backward_noalloc.argtypes = [ctypes.POINTER(dendsn_config)] + \
@@ -175,7 +214,12 @@ def _xdtype(cfg) -> torch.dtype:
 
 def _check_shapes(cfg, x, alpha, xi, zeta, kappa, mask):
     T, B, N, K, C, Kb = cfg.T, cfg.B, cfg.N, cfg.K, cfg.C, cfg.K // cfg.G
-    if tuple(x.shape) != (T, B, N, K) or x.dtype != _xdtype(cfg):
+    if cfg.layout == LAYOUT_PAPER:
+        # [T, B, N / inner, K, inner] in any contiguous shape with that element order
+        if x.numel() != T * B * N * K or x.dtype != _xdtype(cfg) or x.dim() < 2 or \
+                tuple(x.shape[:2]) != (T, B):
+            raise ValueError(f"x must be {_xdtype(cfg)} [{T},{B},...] with {T * B * N * K} elements")
+    elif tuple(x.shape) != (T, B, N, K) or x.dtype != _xdtype(cfg):
         raise ValueError(f"x must be {_xdtype(cfg)} [{T},{B},{N},{K}], got {x.dtype} {tuple(x.shape)}")
     for name, t, shp in (("alpha", alpha, (C, K)), ("xi", xi, (C, K)), ("zeta", zeta, (C, Kb)),
                          ("kappa", kappa, (C, Kb))):
@@ -199,8 +243,9 @@ def workspace(cfg, device=None):
 def forward(cfg, x, alpha, xi, zeta, kappa, mask=None, want_v=False, saved=None, stream=None):
     """Allocating forward. Returns (spikes, v or None)."""
     _check_shapes(cfg, x, alpha, xi, zeta, kappa, mask)
-    spikes = torch.empty(x.shape[:3], dtype=x.dtype, device=x.device)
-    v = torch.empty(x.shape[:3], dtype=torch.float32, device=x.device) if want_v else None
+    shape = (cfg.T, cfg.B, cfg.N)
+    spikes = torch.empty(shape, dtype=x.dtype, device=x.device)
+    v = torch.empty(shape, dtype=torch.float32, device=x.device) if want_v else None
     dendsn_forward(cfg, x, alpha, xi, zeta, kappa, mask, spikes, v, saved, stream)
     return spikes, v
 

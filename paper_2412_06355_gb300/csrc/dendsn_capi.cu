@@ -70,6 +70,7 @@ struct Plan {
     int blocks_f, blocks_b;
     size_t saved_bytes, scratch_bytes, ck_vd_bytes;
     int sx;            // bytes per x element
+    int layout;        // 0 compartments innermost, 1 the paper's layer layout
 };
 
 int sm_count() {
@@ -122,7 +123,7 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) 
     if (!(c.x_dtype == DENDSN_F32 || c.x_dtype == DENDSN_BF16))
         return fail(DENDSN_ERR_INVALID_ARG, "bad x_dtype %d", c.x_dtype);
     if (!is01(c.psi) || !is01(c.reset) || !is01(c.detach_reset) || !is01(c.mask_per_neuron) ||
-        !is01(c.stateless) || !is01(c.residual))
+        !is01(c.stateless) || !is01(c.residual) || !is01(c.layout))
         return fail(DENDSN_ERR_INVALID_ARG, "enum/flag field out of range");
     if (c.surrogate != DENDSN_SG_ATAN)
         return fail(c.surrogate < 0 ? DENDSN_ERR_INVALID_ARG : DENDSN_ERR_UNSUPPORTED,
@@ -166,6 +167,7 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) 
     pl->blocks_f = (int)bf;
     pl->blocks_b = (int)bb;
     pl->sx = (c.x_dtype == DENDSN_BF16) ? 2 : 4;
+    pl->layout = (c.K > 1) ? c.layout : 0;
     const size_t NP = 2 * (size_t)c.K + 2 * (size_t)g.Kb;
     pl->scratch_bytes = (size_t)bb * pl->gb.nch_max * NP * sizeof(float);
     pl->scratch_bytes = (pl->scratch_bytes + 15) / 16 * 16;
@@ -203,42 +205,47 @@ dendsn_status check_params(const float *alpha, const float *xi, const float *zet
     return DENDSN_OK;
 }
 
-#define DENDSN_FWD_CASE(KK, GG)                                                       \
-    if (cfg.K == KK && cfg.G == GG) {                                                 \
-        switch (cfg.psi * 2 + cfg.x_dtype) {                                        \
-        case 0: return launch_forward<KK, GG, 0, 0>(a, blocks, s);                    \
-        case 1: return launch_forward<KK, GG, 0, 1>(a, blocks, s);                    \
-        case 2: return launch_forward<KK, GG, 1, 0>(a, blocks, s);                    \
-        default: return launch_forward<KK, GG, 1, 1>(a, blocks, s);                   \
-        }                                                                           \
+#define DENDSN_FWD_CASE(KK, GG)                                                         \
+    if (cfg.K == KK && cfg.G == GG) {                                                   \
+        switch ((cfg.psi * 2 + cfg.x_dtype) * 2 + layout) {                             \
+        case 0: return launch_forward<KK, GG, 0, 0, 0>(a, blocks, s);                   \
+        case 1: return launch_forward<KK, GG, 0, 0, 1>(a, blocks, s);                   \
+        case 2: return launch_forward<KK, GG, 0, 1, 0>(a, blocks, s);                   \
+        case 3: return launch_forward<KK, GG, 0, 1, 1>(a, blocks, s);                   \
+        case 4: return launch_forward<KK, GG, 1, 0, 0>(a, blocks, s);                   \
+        case 5: return launch_forward<KK, GG, 1, 0, 1>(a, blocks, s);                   \
+        case 6: return launch_forward<KK, GG, 1, 1, 0>(a, blocks, s);                   \
+        default: return launch_forward<KK, GG, 1, 1, 1>(a, blocks, s);                  \
+        }                                                                               \
     }
 
-cudaError_t dispatch_forward(const dendsn_config &cfg, const FwdArgs &a, int blocks,
+// layout: 0 compartments innermost, 1 the paper's layer layout (same as 0 when K = 1)
+cudaError_t dispatch_forward(const dendsn_config &cfg, int layout, const FwdArgs &a, int blocks,
                              cudaStream_t s) {
     DENDSN_KG_LIST(DENDSN_FWD_CASE)
     return cudaErrorInvalidValue;
 }
 
-#define DENDSN_BWD_CASE(KK, GG)                                                       \
-    if (cfg.K == KK && cfg.G == GG) {                                                 \
-        if (L == 4) {                                                               \
-            switch (cfg.psi * 2 + cfg.x_dtype) {                                    \
-            case 0: return launch_backward<KK, GG, 0, 0, 4>(a, blocks, s);            \
-            case 1: return launch_backward<KK, GG, 0, 1, 4>(a, blocks, s);            \
-            case 2: return launch_backward<KK, GG, 1, 0, 4>(a, blocks, s);            \
-            default: return launch_backward<KK, GG, 1, 1, 4>(a, blocks, s);           \
-            }                                                                       \
-        }                                                                           \
-        switch (cfg.psi * 2 + cfg.x_dtype) {                                        \
-        case 0: return launch_backward<KK, GG, 0, 0, 8>(a, blocks, s);                \
-        case 1: return launch_backward<KK, GG, 0, 1, 8>(a, blocks, s);                \
-        case 2: return launch_backward<KK, GG, 1, 0, 8>(a, blocks, s);                \
-        default: return launch_backward<KK, GG, 1, 1, 8>(a, blocks, s);               \
-        }                                                                           \
+#define DENDSN_BWD_L(KK, GG, LL)                                                        \
+    switch ((cfg.psi * 2 + cfg.x_dtype) * 2 + layout) {                                 \
+    case 0: return launch_backward<KK, GG, 0, 0, LL, 0>(a, blocks, s);                  \
+    case 1: return launch_backward<KK, GG, 0, 0, LL, 1>(a, blocks, s);                  \
+    case 2: return launch_backward<KK, GG, 0, 1, LL, 0>(a, blocks, s);                  \
+    case 3: return launch_backward<KK, GG, 0, 1, LL, 1>(a, blocks, s);                  \
+    case 4: return launch_backward<KK, GG, 1, 0, LL, 0>(a, blocks, s);                  \
+    case 5: return launch_backward<KK, GG, 1, 0, LL, 1>(a, blocks, s);                  \
+    case 6: return launch_backward<KK, GG, 1, 1, LL, 0>(a, blocks, s);                  \
+    default: return launch_backward<KK, GG, 1, 1, LL, 1>(a, blocks, s);                 \
     }
 
-cudaError_t dispatch_backward(const dendsn_config &cfg, int L, const BwdArgs &a, int blocks,
-                              cudaStream_t s) {
+#define DENDSN_BWD_CASE(KK, GG)                                                         \
+    if (cfg.K == KK && cfg.G == GG) {                                                   \
+        if (L == 4) { DENDSN_BWD_L(KK, GG, 4) }                                         \
+        DENDSN_BWD_L(KK, GG, 8)                                                         \
+    }
+
+cudaError_t dispatch_backward(const dendsn_config &cfg, int layout, int L, const BwdArgs &a,
+                              int blocks, cudaStream_t s) {
     DENDSN_KG_LIST(DENDSN_BWD_CASE)
     return cudaErrorInvalidValue;
 }
@@ -280,7 +287,7 @@ dendsn_status dendsn_forward(const dendsn_config *cfg, const void *x, const floa
     a.ck_vd = (saved && pl.gf.n_ck > 0) ? static_cast<float *>(saved) : nullptr;
     a.ck_vs = a.ck_vd ? reinterpret_cast<float *>(static_cast<char *>(saved) + pl.ck_vd_bytes)
                       : nullptr;
-    cudaError_t e = dispatch_forward(*cfg, a, pl.blocks_f, static_cast<cudaStream_t>(stream));
+    cudaError_t e = dispatch_forward(*cfg, pl.layout, a, pl.blocks_f, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess)
         return fail(DENDSN_ERR_CUDA, "forward launch failed: %s", cudaGetErrorString(e));
     g_launches.fetch_add(1, std::memory_order_relaxed);
@@ -330,7 +337,7 @@ dendsn_status dendsn_backward(const dendsn_config *cfg, const void *x, const flo
                                 : nullptr;
         a.gx = grad_x;
         a.partials = static_cast<float *>(scratch);
-        cudaError_t e = dispatch_backward(*cfg, pl.gb.L, a, pl.blocks_b, s);
+        cudaError_t e = dispatch_backward(*cfg, pl.layout, pl.gb.L, a, pl.blocks_b, s);
         if (e != cudaSuccess)
             return fail(DENDSN_ERR_CUDA, "backward launch failed: %s", cudaGetErrorString(e));
         g_launches.fetch_add(1, std::memory_order_relaxed);

@@ -650,18 +650,92 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" :: "n"(N) : "memory"); }
 
+// ---------------------------------------------------------------- lane input access
+// LAYOUT 0: x is [T, B, N, K], a neuron's K compartments contiguous (one vector per lane).
+// LAYOUT 1: the paper's layer layout [T, B, N / inner, K, inner] (channels C_o, then
+//           compartments P, then the spatial positions), compartments `inner` apart; a
+//           warp of consecutive neurons reads each compartment as one contiguous span.
+template <typename XT, int KT, int LAYOUT> struct XIO;
+
+template <typename XT, int KT> struct XIO<XT, KT, 0> {
+    using Raw = typename Vec<XT, KT>::Raw;
+    static constexpr bool kAsync = sizeof(Raw) >= 4;
+    static __device__ __forceinline__ Raw load(const XT *p, int64_t) { return Vec<XT, KT>::load(p); }
+    static __device__ __forceinline__ void unpack(const Raw &r, float (&v)[KT]) { Vec<XT, KT>::unpack(r, v); }
+    static __device__ __forceinline__ void store(XT *p, int64_t, const float (&v)[KT]) { Vec<XT, KT>::store(p, v); }
+    static __device__ __forceinline__ void copy_async(Raw *slot, const XT *p, int64_t, float dep) {
+        cp_async_raw(slot, p, dep);
+    }
+};
+
+template <int KT> struct XIO<float, KT, 1> {
+    using Raw = typename Vec<float, KT>::Raw;
+    static constexpr bool kAsync = true;
+    static __device__ __forceinline__ Raw load(const float *p, int64_t ks) {
+        float v[KT];
+#pragma unroll
+        for (int k = 0; k < KT; ++k) v[k] = __ldcs(p + k * ks);
+        return Vec<float, KT>::pack(v);
+    }
+    static __device__ __forceinline__ void unpack(const Raw &r, float (&v)[KT]) { Vec<float, KT>::unpack(r, v); }
+    static __device__ __forceinline__ void store(float *p, int64_t ks, const float (&v)[KT]) {
+#pragma unroll
+        for (int k = 0; k < KT; ++k) __stcs(p + k * ks, v[k]);
+    }
+    static __device__ __forceinline__ void copy_async(Raw *slot, const float *p, int64_t ks, float dep) {
+#pragma unroll
+        for (int k = 0; k < KT; ++k) cp_async<4>(reinterpret_cast<float *>(slot) + k, p + k * ks, dep);
+    }
+};
+
+template <int KT> struct XIO<__nv_bfloat16, KT, 1> {
+    using T = __nv_bfloat16;
+    using Raw = typename Vec<T, KT>::Raw;        // kept packed, as in the contiguous layout
+    static constexpr bool kAsync = false;        // 2-byte elements: no cp.async
+    static __device__ __forceinline__ uint32_t ld16(const T *p) {
+        return __ldcs(reinterpret_cast<const unsigned short *>(p));
+    }
+    static __device__ __forceinline__ uint32_t ld2(const T *p, int64_t ks) {
+        return ld16(p) | (ld16(p + ks) << 16);
+    }
+    static __device__ __forceinline__ Raw load(const T *p, int64_t ks) {
+        if constexpr (KT == 8)
+            return make_uint4(ld2(p, ks), ld2(p + 2 * ks, ks), ld2(p + 4 * ks, ks), ld2(p + 6 * ks, ks));
+        else if constexpr (KT == 4) return make_uint2(ld2(p, ks), ld2(p + 2 * ks, ks));
+        else if constexpr (KT == 2) return ld2(p, ks);
+        else return (unsigned short)ld16(p);
+    }
+    static __device__ __forceinline__ void unpack(const Raw &r, float (&v)[KT]) { Vec<T, KT>::unpack(r, v); }
+    static __device__ __forceinline__ void store(T *p, int64_t ks, const float (&v)[KT]) {
+#pragma unroll
+        for (int k = 0; k < KT; ++k) {
+            __nv_bfloat16 h = __float2bfloat16_rn(v[k]);
+            __stcs(reinterpret_cast<unsigned short *>(p + k * ks), *reinterpret_cast<unsigned short *>(&h));
+        }
+    }
+    static __device__ __forceinline__ void copy_async(Raw *, const T *, int64_t, float) {}
+};
+
+// Offset of lane `sub`'s first compartment of neuron j (steps add T-multiples of B*N*K).
+template <int LAYOUT>
+__device__ __forceinline__ int64_t lane_x_offset(int64_t j, int sub, int KT, int K, int inner) {
+    if constexpr (LAYOUT == 0) return j * K + (int64_t)sub * KT;
+    const int64_t s = j % inner;
+    return (j - s) * K + s + (int64_t)sub * KT * inner;
+}
+
 // x is prefetched kFwdBatch steps ahead of use (a ring of kFwdBatch registers);
 // checkpoints every g.L steps (g.L is a power of two and a multiple of the batch).
-template <int K, int G, int PSI, typename XT>
+template <int K, int G, int PSI, typename XT, int LAYOUT>
 __global__ void __launch_bounds__(fwd_threads(K), lane_compartments(K) >= 8 ? 2 : DENDSN_FWD_MINB)
 dendsn_forward_kernel(const FwdArgs A) {
     constexpr int NT = fwd_threads(K);
     constexpr int KT = lane_compartments(K);
     constexpr int LPN = K / KT;
     constexpr int L = kFwdBatch;
-    using V = Vec<XT, KT>;
+    using V = XIO<XT, KT, LAYOUT>;
     using AR = Arith<KT, G, PSI, XT>;
-    constexpr bool ASYNC = DENDSN_FWD_ASYNC && sizeof(typename V::Raw) >= 4;
+    constexpr bool ASYNC = DENDSN_FWD_ASYNC && V::kAsync;
     const Geometry &g = A.g;
     const Params &P = A.p;
     const ThreadPos pos = thread_pos<LPN>(g);
@@ -676,7 +750,9 @@ dendsn_forward_kernel(const FwdArgs A) {
     const int64_t j0 = pos.row0 * g.P + pos.p;   // first neuron of this thread
     const int64_t jstep = (int64_t)pos.rstride * g.P;
     const int64_t rX = jstep * K;                // x elements between this thread's rows
-    const XT *__restrict__ xrow = static_cast<const XT *>(A.x) + j0 * K + pos.sub * KT;
+    const int64_t ks = LAYOUT == 0 ? 1 : g.inner;   // distance between a lane's compartments
+    const XT *__restrict__ xrow = static_cast<const XT *>(A.x) +
+                                  lane_x_offset<LAYOUT>(j0, pos.sub, KT, K, g.inner);
     XT *__restrict__ srow = static_cast<XT *>(A.spikes) + j0;
     float *vrow = A.v_out ? A.v_out + j0 : nullptr;
     const bool write_ck = (A.ck_vd != nullptr) && g.n_ck > 0 && pos.active;
@@ -696,7 +772,7 @@ dendsn_forward_kernel(const FwdArgs A) {
         const int64_t row_jump = rX - (int64_t)T * sX;
 #pragma unroll
         for (int k = 0; k < D; ++k) {
-            if (ir < pos.nrows) cp_async_raw(ring + k * NT, ip, 0.f);
+            if (ir < pos.nrows) V::copy_async(ring + k * NT, ip, ks, 0.f);
             cp_async_commit();
             ip += sX;
             if (++it == T) { it = 0; ++ir; ip += row_jump; }
@@ -731,10 +807,10 @@ dendsn_forward_kernel(const FwdArgs A) {
                     const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
                     // the slot's value has been used (z depends on it): refill it
                     if constexpr (DIV) {
-                        if (fetch_row) cp_async_raw(ring + slot * NT, cp + ahead, z);
+                        if (fetch_row) V::copy_async(ring + slot * NT, cp + ahead, ks, z);
                         cp += sX;
                     } else {
-                        if (ir < pos.nrows) cp_async_raw(ring + slot * NT, ip, z);
+                        if (ir < pos.nrows) V::copy_async(ring + slot * NT, ip, ks, z);
                         ip += sX;
                         if (++it == T) { it = 0; ++ir; ip += row_jump; }
                     }
@@ -785,7 +861,7 @@ dendsn_forward_kernel(const FwdArgs A) {
         const XT *p = xrow;
 #pragma unroll
         for (int tt = 0; tt < L; ++tt) {
-            if (tt < T) xb[tt] = V::load(p);
+            if (tt < T) xb[tt] = V::load(p, ks);
             p += sX;
         }
     }
@@ -811,7 +887,7 @@ dendsn_forward_kernel(const FwdArgs A) {
                 float xv[KT];
                 V::unpack(xb[tt], xv);
                 // refill slot tt right after its value is taken
-                if (tt < nnext) xb[tt] = V::load(xn);
+                if (tt < nnext) xb[tt] = V::load(xn, ks);
                 xn += sX;
                 if (tt < ncur) {
                     const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
@@ -844,7 +920,7 @@ dendsn_forward_kernel(const FwdArgs A) {
 template <int KT, int G>
 constexpr int acc_count() { return 2 * KT + 2 * (KT / G); }
 
-template <int K, int G, int PSI, typename XT, int L>
+template <int K, int G, int PSI, typename XT, int L, int LAYOUT>
 __global__ void __launch_bounds__(bwd_threads(bwd_lane_compartments(K, G, xt_code<XT>(), L)),
                                   bwd_threads(bwd_lane_compartments(K, G, xt_code<XT>(), L)) == 128 ? 3 : 2)
 dendsn_backward_kernel(const BwdArgs A) {
@@ -859,7 +935,7 @@ dendsn_backward_kernel(const BwdArgs A) {
     // 8-compartment lanes (registers), else in registers
     constexpr bool SHIST = MULTI || KT >= 8;
     constexpr int H = 4;                         // prefetch distance of x in steps
-    using V = Vec<XT, KT>;
+    using V = XIO<XT, KT, LAYOUT>;
     using S1 = Scalar<XT>;
     using AR = Arith<KT, G, PSI, XT>;
     using HistRaw = typename Vec<float, KT>::Raw;
@@ -867,7 +943,7 @@ dendsn_backward_kernel(const BwdArgs A) {
     // x staged through a per-thread cp.async ring in shared memory when the history is
     // there too; otherwise (T <= 4, up to 4 compartments) a register ring, which
     // measured faster there
-    constexpr bool BASYNC = DENDSN_BWD_ASYNC && SHIST && sizeof(XRaw) >= 4;
+    constexpr bool BASYNC = DENDSN_BWD_ASYNC && SHIST && V::kAsync;
     constexpr int D = kBwdDepth;
     const Geometry &g = A.g;
     const Params &P = A.p;
@@ -882,9 +958,11 @@ dendsn_backward_kernel(const BwdArgs A) {
     const int64_t j0 = pos.row0 * g.P + pos.p;
     const int64_t jstep = (int64_t)pos.rstride * g.P;
     const int64_t rX = jstep * K;
-    const XT *__restrict__ xrow = static_cast<const XT *>(A.x) + j0 * K + pos.sub * KT;
+    const int64_t ks = LAYOUT == 0 ? 1 : g.inner;   // distance between a lane's compartments
+    const int64_t xoff = lane_x_offset<LAYOUT>(j0, pos.sub, KT, K, g.inner);
+    const XT *__restrict__ xrow = static_cast<const XT *>(A.x) + xoff;
     const XT *__restrict__ gsrow = static_cast<const XT *>(A.gs) + j0;
-    XT *__restrict__ gxrow = static_cast<XT *>(A.gx) + j0 * K + pos.sub * KT;
+    XT *__restrict__ gxrow = static_cast<XT *>(A.gx) + xoff;
     const float *gvrow = A.gv ? A.gv + j0 : nullptr;
     // dV[t+1]/dS[t] = kv V[t] + cs: hard -beta V[t], soft -beta theta, 0 when detached;
     // dV[t+1]/dV[t] = beta, or b_spike after a spike (0 hard, beta soft)
@@ -917,7 +995,7 @@ dendsn_backward_kernel(const BwdArgs A) {
     if constexpr (BASYNC) {
 #pragma unroll
         for (int k = 0; k < D; ++k) {
-            if (wr < pos.nrows) cp_async_raw(xring + k * NT, wp, 0.f);
+            if (wr < pos.nrows) V::copy_async(xring + k * NT, wp, ks, 0.f);
             cp_async_commit();
             walk();
         }
@@ -939,7 +1017,7 @@ dendsn_backward_kernel(const BwdArgs A) {
 #pragma unroll
         for (int tt = 0; tt < L; ++tt) {
             if (t0 + tt < T) {
-                if (!BASYNC && tt < H) xb[(!BASYNC && tt < H) ? tt : 0] = V::load(p);
+                if (!BASYNC && tt < H) xb[(!BASYNC && tt < H) ? tt : 0] = V::load(p, ks);
                 gsb[tt] = S1::load(q);
             }
             p += sX;
@@ -1009,10 +1087,10 @@ dendsn_backward_kernel(const BwdArgs A) {
                         // refill the slot with the step H ahead: later in this chunk, or
                         // the first steps of the next chunk
                         if (tt + H < L) {
-                            if (tt + H < ncur) xb[BASYNC ? 0 : tt % H] = V::load(xa);
+                            if (tt + H < ncur) xb[BASYNC ? 0 : tt % H] = V::load(xa, ks);
                             xa += sX;
                         } else {
-                            if (tt + H - L < nnext) xb[BASYNC ? 0 : tt % H] = V::load(xnn);
+                            if (tt + H - L < nnext) xb[BASYNC ? 0 : tt % H] = V::load(xnn, ks);
                             xnn += sX;
                         }
                     }
@@ -1024,7 +1102,7 @@ dendsn_backward_kernel(const BwdArgs A) {
                         const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
                         if constexpr (BASYNC) {
                             // the slot's value has been used (z depends on it): refill it
-                            if (wr < pos.nrows) cp_async_raw(xring + xslot * NT, wp, z);
+                            if (wr < pos.nrows) V::copy_async(xring + xslot * NT, wp, ks, z);
                             cp_async_commit();
                             walk();
                             xslot = (xslot == D - 1) ? 0 : xslot + 1;
@@ -1086,7 +1164,7 @@ dendsn_backward_kernel(const BwdArgs A) {
                     if (has_gv) dv = __fadd_rn(dv, __ldcs(gvp));
                     float gxv[KT];
                     AR::backward(lp, vdt, vdp, dv, Ad, acc, residual ? __fmul_rn(dv, inv_k) : 0.f, gxv);
-                    if (pos.active) V::store(gxp, gxv);
+                    if (pos.active) V::store(gxp, ks, gxv);
                     dvn = dv;
                 }
                 gxp -= sX;
@@ -1155,20 +1233,21 @@ cudaError_t allow_smem(Kern kernel, size_t bytes) {
     return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
 }
 
-template <int K, int G, int PSI, int XT>
+template <int K, int G, int PSI, int XT, int LAYOUT>
 cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s) {
     using T = typename XType<XT>::type;
     constexpr int KT = lane_compartments(K);
-    constexpr size_t raw = sizeof(typename Vec<T, KT>::Raw);
+    using XI = XIO<T, KT, LAYOUT>;
+    constexpr size_t raw = sizeof(typename XI::Raw);
     constexpr int NT = fwd_threads(K);
-    const size_t smem = (DENDSN_FWD_ASYNC && raw >= 4) ? raw * kFwdDepth * NT : 0;
-    cudaError_t e = allow_smem(dendsn_forward_kernel<K, G, PSI, T>, smem);
+    const size_t smem = (DENDSN_FWD_ASYNC && XI::kAsync) ? raw * kFwdDepth * NT : 0;
+    cudaError_t e = allow_smem(dendsn_forward_kernel<K, G, PSI, T, LAYOUT>, smem);
     if (e != cudaSuccess) return e;
-    dendsn_forward_kernel<K, G, PSI, T><<<blocks, NT, smem, s>>>(a);
+    dendsn_forward_kernel<K, G, PSI, T, LAYOUT><<<blocks, NT, smem, s>>>(a);
     return cudaGetLastError();
 }
 
-template <int K, int G, int PSI, int XT, int L>
+template <int K, int G, int PSI, int XT, int L, int LAYOUT>
 cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
     using T = typename XType<XT>::type;
     constexpr int KT = bwd_lane_compartments(K, G, XT, L);
@@ -1176,12 +1255,13 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
     const size_t red = sizeof(float) * acc_count<KT, G>() * NT;
     constexpr bool shist = (L > 4) || KT >= 8;
     const size_t hist = shist ? sizeof(float) * (KT + 1) * L * NT : 0;
-    constexpr size_t xraw = sizeof(typename Vec<T, KT>::Raw);
-    const size_t ring = (DENDSN_BWD_ASYNC && shist && xraw >= 4) ? xraw * kBwdDepth * NT : 0;
+    using XI = XIO<T, KT, LAYOUT>;
+    constexpr size_t xraw = sizeof(typename XI::Raw);
+    const size_t ring = (DENDSN_BWD_ASYNC && shist && XI::kAsync) ? xraw * kBwdDepth * NT : 0;
     const size_t smem = red > hist + ring ? red : hist + ring;
-    cudaError_t e = allow_smem(dendsn_backward_kernel<K, G, PSI, T, L>, smem);
+    cudaError_t e = allow_smem(dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT>, smem);
     if (e != cudaSuccess) return e;
-    dendsn_backward_kernel<K, G, PSI, T, L><<<blocks, NT, smem, s>>>(a);
+    dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT><<<blocks, NT, smem, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -79,10 +79,11 @@ struct FinArgs {
     int32_t stateless;
 };
 
-// XT: 0 = float, 1 = bfloat16. Defined in the instantiation units.
-template <int K, int G, int PSI, int XT>
+// XT: 0 = float, 1 = bfloat16. LAYOUT: 0 = compartments innermost, 1 = the paper's
+// (C_o, P, H, W) layer layout. Defined in the instantiation units.
+template <int K, int G, int PSI, int XT, int LAYOUT>
 cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s);
-template <int K, int G, int PSI, int XT, int L>
+template <int K, int G, int PSI, int XT, int L, int LAYOUT>
 cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s);
 cudaError_t launch_finalize(const FinArgs &a, cudaStream_t s);
 

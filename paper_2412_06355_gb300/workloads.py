@@ -5,7 +5,9 @@ the layer workloads; it holds none of the neuron's arithmetic. Both the CUDA pat
 and the CPU oracle are fed from it, so they see identical bits.
 
 Layout (the library's ABI):
-  x      [T, B, N, K]   branch/compartment input currents, K innermost
+  x      [T, B, N, K]   branch/compartment input currents, K innermost; or, for
+                        layout "paper", [T, B, N / inner, K, inner]: a conv layer's
+                        output read as (C_o, P, H, W) with inner = H * W
   alpha  [C, K]         compartment decay factors           (Eq. methods-compartment)
   xi     [C, K]         translation factors                 (Eq. methods-branch-aggregation)
   zeta   [C, Kb]        dilation factors, Kb = K / G        (Eq. methods-branch-aggregation)
@@ -52,6 +54,7 @@ class Workload:
     stateless: bool = False
     residual: bool = False
     detach_reset: bool = False
+    layout: str = "kinner"          # "kinner" [T,B,N,K] or "paper" [T,B,N/inner,K,inner]
     seed: int = 0
 
     @property
@@ -99,6 +102,9 @@ WORKLOADS = {
     "event": Workload("event", T=64, B=32, N=131072, K=4, G=1, C=128, inner=1024,
                       dtype="f32", psi="mh", reset="hard", x_mean=0.8, x_std=1.0,
                       x_density=0.2, seed=3),
+    "conv_paper_p4b2": Workload("conv_paper_p4b2", T=4, B=64, N=131072, K=4, G=2, C=128,
+                                inner=1024, dtype="f32", psi="mh", reset="hard",
+                                layout="paper", seed=5),
     "token_dbg": Workload("token_dbg", T=4, B=64, N=196 * 384, K=8, G=1, C=384, inner=1,
                           dtype="f32", psi="mh", reset="hard", mask_p=0.5,
                           mask_per_neuron=True, seed=4),
@@ -127,6 +133,8 @@ def make_inputs(w: Workload, device: str = "cpu", with_gv: bool = False) -> dict
         x.mul_(keep)
         del keep
     x = x.to(torch_dtype(w))
+    if w.layout == "paper":
+        x = to_paper_layout(x, w.inner)
     alpha = torch.rand((C, K), generator=g, **f32).mul_(0.45).add_(0.5)
     xi = torch.randn((C, K), generator=g, **f32).mul_(0.1)
     zeta = torch.rand((C, Kb), generator=g, **f32).mul_(0.4).add_(0.8)
@@ -138,6 +146,18 @@ def make_inputs(w: Workload, device: str = "cpu", with_gv: bool = False) -> dict
     gs = torch.randn((T, B, N), generator=g, **f32).to(torch_dtype(w))
     gv = torch.randn((T, B, N), generator=g, **f32) if with_gv else None
     return dict(x=x, alpha=alpha, xi=xi, zeta=zeta, kappa=kappa, mask=mask, gs=gs, gv=gv)
+
+
+def to_paper_layout(x: torch.Tensor, inner: int) -> torch.Tensor:
+    """[T, B, N, K] -> the paper's [T, B, N / inner, K, inner] (a pure permutation)."""
+    T, B, N, K = x.shape
+    return x.reshape(T, B, N // inner, inner, K).permute(0, 1, 2, 4, 3).contiguous()
+
+
+def from_paper_layout(x: torch.Tensor, N: int, K: int, inner: int) -> torch.Tensor:
+    """The paper's [T, B, N / inner, K, inner] -> [T, B, N, K] (a pure permutation)."""
+    T, B = x.shape[:2]
+    return x.reshape(T, B, N // inner, K, inner).permute(0, 1, 2, 4, 3).reshape(T, B, N, K)
 
 
 def scaled(w: Workload, B: Optional[int] = None, N: Optional[int] = None,

@@ -134,6 +134,29 @@ def test_null_and_misaligned_pointers_rejected_before_launch(lib):
     assert st == 1 and b"checkpoints" in lib.dendsn_last_error()
 
 
+def test_layout_flag_validated():
+    cfg = make_config(T=4, B=2, N=64, K=4, C=4, inner=16, layout="paper")
+    assert cfg.layout == binding.LAYOUT_PAPER
+    assert status_of(binding.dendsn_workspace_size, cfg) == 0
+    cfg.layout = 2
+    assert status_of(binding.dendsn_workspace_size, cfg) == 1
+
+
+def test_binding_refuses_undersized_tensors(lib):
+    """Sizes are checked on the host before any pointer reaches the library."""
+    import torch
+    cfg = make_config(T=4, B=2, N=64, K=4, C=4, inner=16, layout="paper")
+    x = torch.zeros(4, 2, 4, 4, 16)                       # the paper layout: right size
+    p = [torch.zeros(4, 4) for _ in range(4)]
+    with pytest.raises(ValueError, match="spikes"):
+        binding.dendsn_forward(cfg, x, *p, None, torch.zeros(4, 2, 4))   # [T, B, N/inner]
+    with pytest.raises(ValueError, match="x:"):
+        binding.dendsn_forward(cfg, x[:, :1], *p, None, torch.zeros(4, 2, 64))
+    with pytest.raises(ValueError, match="scratch"):
+        binding.dendsn_backward(cfg, x, *p, None, torch.zeros(4, 2, 64), None, None,
+                                torch.zeros_like(x), *p, torch.zeros(1))
+
+
 def test_status_strings(lib):
     for code in range(5):
         assert lib.dendsn_status_string(code)

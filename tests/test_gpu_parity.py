@@ -38,6 +38,8 @@ SCALED = {
     "deepconv_bf16": scaled(WORKLOADS["deepconv_bf16"], B=2),
     "event": WORKLOADS["event"].with_(C=32, N=32 * 1024, B=2),
     "token_dbg": scaled(WORKLOADS["token_dbg"], B=2),
+    "conv_paper_p4b2": scaled(WORKLOADS["conv_paper_p4b2"], B=2),
+    "deepconv_bf16_paper": scaled(WORKLOADS["deepconv_bf16"], B=2).with_(layout="paper"),
 }
 
 
@@ -53,15 +55,42 @@ KG = [(1, 1), (2, 1), (2, 2), (4, 1), (4, 2), (4, 4), (8, 1), (8, 2), (8, 4),
       (16, 1), (16, 2), (16, 4)]
 
 
+@pytest.mark.parametrize("layout", ["kinner", "paper"])
 @pytest.mark.parametrize("K,G", KG)
-def test_every_compiled_kg(K, G):
+def test_every_compiled_kg(K, G, layout):
     i = KG.index((K, G))
     w = workloads.Workload(
         f"kg{K}_{G}", T=9, B=3, N=35 * 2, K=K, G=G, C=5, inner=7,
         dtype="bf16" if i % 3 == 2 else "f32", psi="mh" if i % 2 == 0 else "identity",
         reset="soft" if i % 4 == 1 else "hard", mask_p=0.6 if i % 2 else None,
-        mask_per_neuron=(i % 4 == 3), seed=100 + i)
+        mask_per_neuron=(i % 4 == 3), layout=layout, seed=100 + i)
     check_layer(w)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("K,G,T", [(2, 2, 3), (4, 2, 4), (4, 1, 12), (8, 1, 4), (8, 2, 9),
+                                   (16, 4, 5)])
+def test_paper_layout_is_bitwise_the_kinner_layer(K, G, T, dtype):
+    """Only the addresses differ between the layouts: every output must be bit-identical."""
+    w = workloads.Workload("lay", T=T, B=3, N=4 * 2 * 40, K=K, G=G, C=4, inner=40,
+                           dtype=dtype, psi="mh", reset="hard", mask_p=0.7, seed=21)
+    wp = w.with_(layout="paper")
+    outs = []
+    for ww in (w, wp):
+        inp = to_dev(workloads.make_inputs(ww, "cpu", with_gv=True))
+        cfg = binding.config_of(ww)
+        saved, scratch = binding.workspace(cfg)
+        s, v = binding.forward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"],
+                               inp["kappa"], inp["mask"], want_v=True, saved=saved)
+        g = binding.backward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"],
+                             inp["kappa"], inp["mask"], inp["gs"], inp["gv"], saved, scratch)
+        outs.append((s, v, g))
+    torch.cuda.synchronize()
+    (s, v, g), (sp, vp, gp) = outs
+    assert torch.equal(s, sp) and torch.equal(v, vp)
+    assert torch.equal(g["gx"], workloads.from_paper_layout(gp["gx"], w.N, w.K, w.inner))
+    for k in ("galpha", "gxi", "gzeta", "gkappa"):
+        assert torch.equal(g[k], gp[k]), k
 
 
 @pytest.mark.parametrize("kw", [
@@ -184,6 +213,15 @@ def sample_neurons(w, count, seed):
     return flat // w.N, flat % w.N
 
 
+def x_of_neurons(w, x, bt, nt):
+    """[T, M, K] compartment values of neurons (bt[m], nt[m]) in either layout."""
+    if w.layout == "paper":
+        x5 = x.reshape(w.T, w.B, w.N // w.inner, w.K, w.inner)
+        # separated advanced indices put the sample axis first: [M, T, K] -> [T, M, K]
+        return x5[:, bt, nt // w.inner, :, nt % w.inner].transpose(0, 1)
+    return x[:, bt, nt, :]
+
+
 FULL = [(n, {}) for n in WORKLOADS] + [
     ("conv", dict(stateless=True, residual=True)),        # ResStateless (the Tiny ImageNet choice)
     ("conv", dict(stateless=True)),                       # Stateless (the CIFAR10-DVS choice)
@@ -200,7 +238,7 @@ def test_full_size_sampled(name, kw):
     bt, nt = torch.from_numpy(b_idx).cuda(), torch.from_numpy(n_idx).cuda()
 
     # oracle on the sampled neurons (independent of the rest of the layer)
-    xs = inp["x"][:, bt, nt, :].cpu()                                  # [T, M, K]
+    xs = x_of_neurons(w, inp["x"], bt, nt).cpu()                       # [T, M, K]
     chan = ((n_idx // w.inner) % w.C).astype(np.int32)
     mrow = (n_idx if w.mask_per_neuron else chan).astype(np.int32)
     ocfg = oracle.OracleConfig(T=w.T, K=w.K, G=w.G, C=w.C, psi=w.psi, reset=w.reset,
@@ -225,7 +263,7 @@ def test_full_size_sampled(name, kw):
     torch.cuda.synchronize()
     got_s = oracle.to_f64(s[:, bt, nt])
     got_v = oracle.to_f64(v[:, bt, nt])
-    got_gx = oracle.to_f64(g["gx"][:, bt, nt, :])
+    got_gx = oracle.to_f64(x_of_neurons(w, g["gx"], bt, nt))
     t_idx = np.arange(w.T)[:, None]
     assert_close("V^s", got_v, v_o, V_RTOL, 0.0, mask=t_idx <= first[None], atol_abs=V_ATOL)
     sm = t_idx < first[None]
@@ -237,6 +275,9 @@ def test_full_size_sampled(name, kw):
     for k in ("galpha", "gxi", "gzeta", "gkappa"):
         assert_close(k, oracle.to_f64(g[k]), ref[k], G_RTOL, G_ATOL_REL)
     # every non-sampled neuron received zero upstream gradient: its grad_x is zero
-    gx_abs = g["gx"].abs().sum(dim=(0, 3))
+    gx = g["gx"]
+    if w.layout == "paper":
+        gx = workloads.from_paper_layout(gx, w.N, w.K, w.inner)
+    gx_abs = gx.abs().sum(dim=(0, 3))
     gx_abs[bt, nt] = 0
     assert torch.count_nonzero(gx_abs).item() == 0

@@ -453,3 +453,40 @@ def test_layer_channel_map():
     chan, mrow = layer_channels(B=2, N=8, C=4, inner=1, mask_per_neuron=True)
     assert chan.tolist() == [0, 1, 2, 3, 0, 1, 2, 3] * 2
     assert mrow.tolist() == list(range(8)) * 2
+
+
+def test_paper_layout_reader_places_each_compartment():
+    """(C_o, P, H, W) grouping: compartment k of neuron n = g*inner + s sits at [g, k, s]."""
+    from types import SimpleNamespace
+    from oracle import layer_x
+    T, B, N, K, inner = 2, 2, 6, 2, 3
+    w = SimpleNamespace(T=T, B=B, N=N, K=K, inner=inner, layout="paper")
+    xp = np.zeros((T, B, N // inner, K, inner))
+    for t in range(T):
+        for b in range(B):
+            for g in range(N // inner):
+                for k in range(K):
+                    for s in range(inner):
+                        xp[t, b, g, k, s] = 1000 * t + 100 * b + 10 * (g * inner + s) + k
+    got = layer_x(w, xp).reshape(T, B, N, K)
+    t, b, n, k = np.meshgrid(*[np.arange(d) for d in (T, B, N, K)], indexing="ij")
+    assert np.array_equal(got, 1000 * t + 100 * b + 10 * n + k)
+
+
+def test_paper_layout_gives_the_same_layer():
+    """The same draws in either layout give the same spikes and (permuted) gradients."""
+    from oracle import backward_layer, forward_layer
+    from paper_2412_06355_gb300 import workloads
+    w = workloads.Workload("lay", T=5, B=2, N=2 * 3 * 4, K=4, G=2, C=3, inner=4, dtype="f32",
+                           psi="mh", reset="hard", seed=11)
+    wp = w.with_(layout="paper")
+    a, ap = workloads.make_inputs(w, with_gv=True), workloads.make_inputs(wp, with_gv=True)
+    assert tuple(ap["x"].shape) == (5, 2, 2 * 3, 4, 4)
+    s, v = forward_layer(w, a)
+    sp, vp = forward_layer(wp, ap)
+    assert np.array_equal(s, sp) and np.array_equal(v, vp)
+    g, gp = backward_layer(w, a), backward_layer(wp, ap)
+    gx_back = gp["gx"].transpose(0, 1, 2, 4, 3).reshape(g["gx"].shape)
+    assert np.array_equal(g["gx"], gx_back)
+    for k in ("galpha", "gxi", "gzeta", "gkappa"):
+        assert np.array_equal(g[k], gp[k])
