@@ -319,3 +319,93 @@ int oracle_backward(const oracle_cfg *cfg, const double *x, const int32_t *chan,
     free(work);
     return 0;
 }
+
+/*
+ * Point-neuron LIF layer: the soma of the DendSN (Eq. methods-lif-reset-charge,
+ * Eq. methods-lif-fire) driven directly by one input current per neuron, i.e. the
+ * LIF neuron the paper's point-neuron SNNs use and compares its speed against
+ * (Results, "Dendritic spiking neural networks" efficiency paragraph):
+ *
+ *   hard  V[t] = beta (1 - S[t-1]) V[t-1] + X[t]
+ *   soft  V[t] = beta (V[t-1] - theta S[t-1]) + X[t]
+ *   fire  S[t] = Theta(V[t] - theta), V[-1] = S[-1] = 0
+ *
+ * Only T, M, reset, detach_reset, smooth_spike, theta and beta of cfg are read.
+ *   x [T][M]; s_out, v_out [T][M] (v_out may be NULL).
+ */
+int oracle_lif_forward(const oracle_cfg *cfg, const double *x, double *s_out, double *v_out)
+{
+    if (cfg == NULL || cfg->T < 0 || cfg->M < 0)
+        return -1;
+    const int T = cfg->T;
+    const int64_t M = cfg->M;
+    for (int64_t m = 0; m < M; ++m) {
+        double v = 0.0, s = 0.0;
+        for (int t = 0; t < T; ++t) {
+            const double xt = x[(int64_t)t * M + m];
+            if (cfg->reset == 0)
+                v = cfg->beta * (1.0 - s) * v + xt;
+            else
+                v = cfg->beta * (v - cfg->theta * s) + xt;
+            s = fire(cfg, v);
+            s_out[(int64_t)t * M + m] = s;
+            if (v_out != NULL)
+                v_out[(int64_t)t * M + m] = v;
+        }
+    }
+    return 0;
+}
+
+/*
+ * BPTT of the LIF layer with the arctan surrogate (Eq. methods-sg): the soma
+ * part of the DendSN backward, with dX[t] = dV[t] since X enters V linearly.
+ *   gs [T][M]; gv [T][M] or NULL; gx [T][M] (overwritten).
+ */
+int oracle_lif_backward(const oracle_cfg *cfg, const double *x, const double *gs,
+                        const double *gv, double *gx)
+{
+    if (cfg == NULL || cfg->T < 0 || cfg->M < 0)
+        return -1;
+    const int T = cfg->T;
+    const int64_t M = cfg->M;
+    double *vt = (double *)malloc(sizeof(double) * 2 * ((size_t)T + 1));
+    if (vt == NULL)
+        return -1;
+    double *st = vt + T + 1;
+    for (int64_t m = 0; m < M; ++m) {
+        /* forward, keeping V[t] and S[t] */
+        double vv = 0.0, ss = 0.0;
+        for (int t = 0; t < T; ++t) {
+            const double in = x[(int64_t)t * M + m];
+            if (cfg->reset == 0)
+                vv = cfg->beta * (1.0 - ss) * vv + in;
+            else
+                vv = cfg->beta * (vv - cfg->theta * ss) + in;
+            ss = fire(cfg, vv);
+            vt[t] = vv;
+            st[t] = ss;
+        }
+        /* reverse time: g_next = dL/dV[t+1] */
+        double g_next = 0.0;
+        for (int t = T - 1; t >= 0; --t) {
+            double a_vv, a_vs;                    /* dV[t+1]/dV[t], dV[t+1]/dS[t] */
+            if (cfg->reset == 0) {
+                a_vv = cfg->beta * (1.0 - st[t]);
+                a_vs = -cfg->beta * vt[t];
+            } else {
+                a_vv = cfg->beta;
+                a_vs = -cfg->beta * cfg->theta;
+            }
+            if (cfg->detach_reset)
+                a_vs = 0.0;
+            const double g_s = gs[(int64_t)t * M + m] + a_vs * g_next;
+            double g_v = surrogate_deriv(vt[t] - cfg->theta) * g_s + a_vv * g_next;
+            if (gv != NULL)
+                g_v += gv[(int64_t)t * M + m];
+            gx[(int64_t)t * M + m] = g_v;         /* V[t] is linear in X[t] */
+            g_next = g_v;
+        }
+    }
+    free(vt);
+    return 0;
+}

@@ -69,7 +69,8 @@ def build(force: bool = False) -> str:
 
 def _configure(lib):
     P = ctypes.c_void_p
-    for name, nargs in (("oracle_forward", 11), ("oracle_backward", 16)):
+    for name, nargs in (("oracle_forward", 11), ("oracle_backward", 16),
+                        ("oracle_lif_forward", 4), ("oracle_lif_backward", 5)):
         fn = getattr(lib, name)
         fn.restype = ctypes.c_int
         fn.argtypes = [ctypes.POINTER(_Cfg)] + [P] * (nargs - 1)
@@ -177,6 +178,52 @@ def backward(c: OracleConfig, x, chan, mrow, alpha, xi, zeta, kappa, mask, gs, g
     if rc != 0:
         raise RuntimeError("oracle_backward failed")
     return out
+
+
+@dataclasses.dataclass
+class LIFConfig:
+    """Point-neuron LIF layer (the DendSN soma driven directly by one current per neuron)."""
+    T: int
+    reset: str = "hard"
+    theta: float = 1.0
+    beta: float = 0.5
+    detach_reset: bool = False
+    smooth_spike: bool = False
+
+
+def _lif_cfg(c: LIFConfig, M: int) -> _Cfg:
+    return _Cfg(c.T, M, 1, 1, 1, 0, 0 if c.reset == "hard" else 1, 0, 0,
+                int(c.detach_reset), int(c.smooth_spike), float(c.theta), float(c.beta))
+
+
+def lif_forward(c: LIFConfig, x):
+    """LIF forward of M neurons. x: [T, M] (or [T, ...]). Returns (S, V) float64, x's shape."""
+    x = to_f64(x)
+    shape = x.shape
+    assert shape[0] == c.T, (shape, c)
+    x = np.ascontiguousarray(x.reshape(c.T, -1))
+    M = x.shape[1]
+    s = np.zeros((c.T, M))
+    v = np.zeros((c.T, M))
+    cfg = _lif_cfg(c, M)
+    if _load().oracle_lif_forward(ctypes.byref(cfg), _ptr(x), _ptr(s), _ptr(v)) != 0:
+        raise RuntimeError("oracle_lif_forward failed")
+    return s.reshape(shape), v.reshape(shape)
+
+
+def lif_backward(c: LIFConfig, x, gs, gv=None):
+    """LIF backward of M neurons; returns dL/dX with x's shape."""
+    x = to_f64(x)
+    shape = x.shape
+    x = np.ascontiguousarray(x.reshape(c.T, -1))
+    M = x.shape[1]
+    gs = np.ascontiguousarray(to_f64(gs).reshape(c.T, M))
+    gv = None if gv is None else np.ascontiguousarray(to_f64(gv).reshape(c.T, M))
+    gx = np.zeros((c.T, M))
+    cfg = _lif_cfg(c, M)
+    if _load().oracle_lif_backward(ctypes.byref(cfg), _ptr(x), _ptr(gs), _ptr(gv), _ptr(gx)) != 0:
+        raise RuntimeError("oracle_lif_backward failed")
+    return gx.reshape(shape)
 
 
 def layer_channels(B: int, N: int, C: int, inner: int, mask_per_neuron: bool):

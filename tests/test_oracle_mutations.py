@@ -13,6 +13,7 @@ import pytest
 
 import oracle
 import oracle.oracle as oracle_mod
+import test_oracle_lif_pins as lif_pins
 import test_oracle_pins as pins
 
 # (id, text in the oracle source, replacement)
@@ -42,6 +43,15 @@ MUTATIONS = [
     ("direct_no_zeta", "direct[i] = du / z_[b];", "direct[i] = du;"),
     ("gv_dropped", "dv += gv[(int64_t)t * M + m];", "dv += 0.0;"),
     ("residual_grad", "g += dz / K;", "g += dz;"),
+    # the point-neuron LIF layer
+    ("lif_reset_dropped", "v = cfg->beta * (1.0 - s) * v + xt;", "v = cfg->beta * v + xt;"),
+    ("lif_soft_theta", "v = cfg->beta * (v - cfg->theta * s) + xt;", "v = cfg->beta * (v - s) + xt;"),
+    ("lif_bwd_recompute_reset", "vv = cfg->beta * (1.0 - ss) * vv + in;", "vv = cfg->beta * vv + in;"),
+    ("lif_bwd_reset_gate", "a_vv = cfg->beta * (1.0 - st[t]);", "a_vv = cfg->beta;"),
+    ("lif_bwd_reset_sign", "a_vs = -cfg->beta * vt[t];", "a_vs = cfg->beta * vt[t];"),
+    ("lif_bwd_soft_theta", "a_vs = -cfg->beta * cfg->theta;", "a_vs = -cfg->beta;"),
+    ("lif_bwd_gv_dropped", "g_v += gv[(int64_t)t * M + m];", "g_v += 0.0;"),
+    ("lif_bwd_no_carry", "g_next = g_v;", "g_next = 0.0;"),
 ]
 
 PIN_TESTS = [
@@ -60,6 +70,13 @@ PIN_TESTS = [
     lambda: pins.test_backward_matches_autograd_restatement(pins.VARIANTS[3]),
     lambda: pins.test_backward_matches_autograd_restatement(pins.VARIANTS[1]),
     lambda: pins.test_backward_matches_autograd_restatement(pins.VARIANTS[7]),
+    lif_pins.test_lif_golden_worked_trajectories,
+    lambda: lif_pins.test_lif_constant_input_geometric_series_and_period(0.3, 0.5),
+    lambda: lif_pins.test_lif_subthreshold_gradient_closed_form("hard", False),
+    lambda: lif_pins.test_lif_smooth_spike_finite_differences("hard", False),
+    lambda: lif_pins.test_lif_smooth_spike_finite_differences("soft", False),
+    *[(lambda a=a: lif_pins.test_lif_backward_matches_autograd_restatement(*a))
+      for a in lif_pins.LIF_AUTOGRAD],
 ]
 
 
