@@ -228,12 +228,17 @@ int oracle_forward(const oracle_cfg *cfg, const double *x, const int32_t *chan,
  *   gx [T][M][K]: dL/dX (overwritten).
  *   galpha, gxi [C][K], gzeta, gkappa [C][Kb]: summed over every neuron of a
  *   channel and every step (overwritten).
+ *   gbeta [C] or NULL: dL/dbeta of the somatic decay, summed the same way, for a
+ *   soma whose beta is learnable (the PLIF soma the paper cites, read as
+ *   Eq. methods-lif-reset-charge with beta a parameter):
+ *     dV^s[t+1]/dbeta = (1 - S[t]) V^s[t]      (hard reset)
+ *                     = V^s[t] - theta S[t]     (soft reset)
  */
 int oracle_backward(const oracle_cfg *cfg, const double *x, const int32_t *chan,
                     const int32_t *mrow, const double *alpha, const double *xi,
                     const double *zeta, const double *kappa, const uint8_t *mask,
                     const double *gs, const double *gv, double *gx, double *galpha,
-                    double *gxi, double *gzeta, double *gkappa)
+                    double *gxi, double *gzeta, double *gkappa, double *gbeta)
 {
     if (cfg == NULL || cfg->K <= 0 || cfg->G <= 0 || cfg->K % cfg->G != 0 || cfg->T < 0)
         return -1;
@@ -243,6 +248,8 @@ int oracle_backward(const oracle_cfg *cfg, const double *x, const int32_t *chan,
     memset(gxi, 0, sizeof(double) * (size_t)cfg->C * K);
     memset(gzeta, 0, sizeof(double) * (size_t)cfg->C * Kb);
     memset(gkappa, 0, sizeof(double) * (size_t)cfg->C * Kb);
+    if (gbeta != NULL)
+        memset(gbeta, 0, sizeof(double) * (size_t)cfg->C);
     double *work = (double *)malloc(sizeof(double) *
                                     ((size_t)(T + 1) * K + 2 * (size_t)T + 2 * (size_t)T * Kb +
                                      4 * (size_t)K + 3 * (size_t)Kb));
@@ -281,6 +288,11 @@ int oracle_backward(const oracle_cfg *cfg, const double *x, const int32_t *chan,
             }
             if (cfg->detach_reset)
                 dvds_next = 0.0;
+            if (gbeta != NULL) {
+                /* beta's direct effect on V^s[t+1] */
+                double leak = (cfg->reset == 0) ? (1.0 - s[t]) * vs[t] : vs[t] - cfg->theta * s[t];
+                gbeta[ch] += dv_next * leak;
+            }
             ds += dvds_next * dv_next;
             double dv = surrogate_deriv(vs[t] - cfg->theta) * ds + dvdv_next * dv_next;
             if (gv != NULL)

@@ -69,7 +69,7 @@ def build(force: bool = False) -> str:
 
 def _configure(lib):
     P = ctypes.c_void_p
-    for name, nargs in (("oracle_forward", 11), ("oracle_backward", 16),
+    for name, nargs in (("oracle_forward", 11), ("oracle_backward", 17),
                         ("oracle_lif_forward", 4), ("oracle_lif_backward", 5)):
         fn = getattr(lib, name)
         fn.restype = ctypes.c_int
@@ -163,18 +163,19 @@ def forward(c: OracleConfig, x, chan, mrow, alpha, xi, zeta, kappa, mask=None):
 
 
 def backward(c: OracleConfig, x, chan, mrow, alpha, xi, zeta, kappa, mask, gs, gv=None):
-    """Backward of M neurons. Returns dict gx [T,M,K], galpha, gxi [C,K], gzeta, gkappa [C,Kb]."""
+    """Backward of M neurons. Returns dict gx [T,M,K], galpha, gxi [C,K], gzeta, gkappa [C,Kb],
+    gbeta [C] (dL/dbeta per channel; a layer-wide beta's gradient is the sum)."""
     x, M, chan, mrow, p, mask = _prep(c, x, chan, mrow, alpha, xi, zeta, kappa, mask)
     gs = to_f64(gs).reshape(c.T, M)
     gv = None if gv is None else to_f64(gv).reshape(c.T, M)
     out = dict(gx=np.zeros((c.T, M, c.K)), galpha=np.zeros((c.C, c.K)),
                gxi=np.zeros((c.C, c.K)), gzeta=np.zeros((c.C, c.Kb)),
-               gkappa=np.zeros((c.C, c.Kb)))
+               gkappa=np.zeros((c.C, c.Kb)), gbeta=np.zeros(c.C))
     cfg = _cfg(c, M)
     rc = _load().oracle_backward(ctypes.byref(cfg), _ptr(x), _ptr(chan), _ptr(mrow),
                                  *[_ptr(a) for a in p], _ptr(mask), _ptr(gs), _ptr(gv),
                                  _ptr(out["gx"]), _ptr(out["galpha"]), _ptr(out["gxi"]),
-                                 _ptr(out["gzeta"]), _ptr(out["gkappa"]))
+                                 _ptr(out["gzeta"]), _ptr(out["gkappa"]), _ptr(out["gbeta"]))
     if rc != 0:
         raise RuntimeError("oracle_backward failed")
     return out

@@ -43,6 +43,12 @@ MUTATIONS = [
     ("direct_no_zeta", "direct[i] = du / z_[b];", "direct[i] = du;"),
     ("gv_dropped", "dv += gv[(int64_t)t * M + m];", "dv += 0.0;"),
     ("residual_grad", "g += dz / K;", "g += dz;"),
+    # the learnable somatic decay (PLIF soma)
+    ("gbeta_hard_leak", "(1.0 - s[t]) * vs[t] : vs[t] - cfg->theta * s[t];",
+     "vs[t] : vs[t] - cfg->theta * s[t];"),
+    ("gbeta_soft_theta", "(1.0 - s[t]) * vs[t] : vs[t] - cfg->theta * s[t];",
+     "(1.0 - s[t]) * vs[t] : vs[t] - s[t];"),
+    ("gbeta_wrong_step", "gbeta[ch] += dv_next * leak;", "gbeta[ch] += gs[(int64_t)t * M + m] * leak;"),
     # the point-neuron LIF layer
     ("lif_reset_dropped", "v = cfg->beta * (1.0 - s) * v + xt;", "v = cfg->beta * v + xt;"),
     ("lif_soft_theta", "v = cfg->beta * (v - cfg->theta * s) + xt;", "v = cfg->beta * (v - s) + xt;"),

@@ -15,6 +15,7 @@ wrong sign or index, a transposed operand) breaks at least one of them:
 * invariants: kappa linearity, masking == zero strength, K identical branches,
   stateless == stateful with alpha = 0, per-channel parameter-gradient sums
 """
+import dataclasses
 import json
 import math
 import os
@@ -251,6 +252,22 @@ def test_backward_matches_finite_differences(var, mode):
             assert np.all(out[name] == 0.0)
             continue
         np.testing.assert_allclose(out[name], g, rtol=1e-6, atol=1e-8, err_msg=name)
+    # the somatic decay (learnable in a PLIF soma): beta is one number shared by every
+    # channel, so finite differences see the sum of the per-channel gradients
+    h = 1e-6
+
+    def L_beta(b):
+        s, v = forward(dataclasses.replace(cfg, beta=b), x, chan, chan, *params, mask)
+        return float((ws * s).sum() + (wv * v).sum())
+
+    fb = (L_beta(cfg.beta + h) - L_beta(cfg.beta - h)) / (2 * h)
+    np.testing.assert_allclose(out["gbeta"].sum(), fb, rtol=1e-6, atol=1e-8)
+    # and each channel's entry collects exactly its own neurons
+    for c in range(C):
+        own = (chan == c)[None, :]
+        oc = backward(cfg, x, chan, chan, *params, mask, ws * own, wv * own)
+        np.testing.assert_allclose(oc["gbeta"][c], out["gbeta"][c], rtol=1e-12, atol=1e-14)
+        assert np.all(np.delete(oc["gbeta"], c) == 0.0)
 
 
 def test_detach_reset_is_not_the_smooth_derivative():
@@ -284,9 +301,11 @@ class _Spike(torch.autograd.Function):
         return g / (1 + (math.pi * x) ** 2)
 
 
-def torch_dendsn(cfg, x, chan, mrow, alpha, xi, zeta, kappa, mask):
+def torch_dendsn(cfg, x, chan, mrow, alpha, xi, zeta, kappa, mask, beta=None):
     """Tensor restatement of the layer (float64 autograd), written independently
-    of the C oracle: tensors over neurons, a Python loop over time."""
+    of the C oracle: tensors over neurons, a Python loop over time. beta: the
+    somatic decay as a tensor (to differentiate it), else cfg.beta."""
+    beta = cfg.beta if beta is None else beta
     T, M, K = x.shape
     Kb, G = cfg.Kb, cfg.G
     a = torch.zeros_like(alpha[chan]) if cfg.stateless else alpha[chan]   # [M, K]
@@ -307,9 +326,9 @@ def torch_dendsn(cfg, x, chan, mrow, alpha, xi, zeta, kappa, mask):
             z = z + x[t].mean(-1)
         sr = sp.detach() if cfg.detach_reset else sp
         if cfg.reset == "hard":
-            vs = cfg.beta * (1 - sr) * vs + z
+            vs = beta * (1 - sr) * vs + z
         else:
-            vs = cfg.beta * (vs - cfg.theta * sr) + z
+            vs = beta * (vs - cfg.theta * sr) + z
         sp = _Spike.apply(vs - cfg.theta)
         S.append(sp)
         V.append(vs)
@@ -336,9 +355,9 @@ def test_backward_matches_autograd_restatement(var):
     out = backward(cfg, x, chan, chan, alpha, xi, zeta, kappa, mask, gs, gv)
 
     tt = lambda a: torch.tensor(a, dtype=torch.float64, requires_grad=True)
-    X, A, XI, Z, KA = map(tt, (x, alpha, xi, zeta, kappa))
+    X, A, XI, Z, KA, BE = map(tt, (x, alpha, xi, zeta, kappa, cfg.beta))
     S, V = torch_dendsn(cfg, X, torch.as_tensor(chan, dtype=torch.long), chan, A, XI, Z, KA,
-                        torch.as_tensor(mask))
+                        torch.as_tensor(mask), beta=BE)
     assert 0.05 < S.mean().item() < 0.95, "case should spike sometimes"
     # spike decisions can only differ where V sits on the threshold to rounding
     assert np.array_equal(S.detach().numpy(), s_o)
@@ -351,6 +370,7 @@ def test_backward_matches_autograd_restatement(var):
     np.testing.assert_allclose(out["gxi"], XI.grad.numpy(), rtol=1e-10, atol=1e-12)
     np.testing.assert_allclose(out["gzeta"], Z.grad.numpy(), rtol=1e-10, atol=1e-12)
     np.testing.assert_allclose(out["gkappa"], KA.grad.numpy(), rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(out["gbeta"].sum(), BE.grad.item(), rtol=1e-10, atol=1e-12)
 
 
 # --------------------------------------------------------------------------- invariants
