@@ -42,6 +42,8 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-lif", action="store_true",
+                    help="skip timing the point-neuron LIF layer baseline")
     ap.add_argument("--workload", default="conv")
     ap.add_argument("--psi", choices=["mh", "identity"], default=None)
     ap.add_argument("--batch", type=int, default=None,
@@ -291,6 +293,43 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def time_lif(T, B, N, dtype, steps, warmup, stream):
+    """Fused LIF layer fwd+bwd (the point-neuron baseline) timed like the DendSN step."""
+    import torch
+    from paper_2412_06355_gb300 import binding, workloads
+    inp = workloads.make_lif_inputs(T, B, N, dtype, seed=11, device="cuda")
+    cfg = binding.make_lif_config(T, B, N, dtype)
+    x, gs = inp["x"], inp["gs"]
+    saved = binding.lif_workspace(cfg)
+    spikes, gx = torch.empty_like(x), torch.empty_like(x)
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        binding.dendsn_lif_forward(cfg, x, spikes, None, saved, stream)
+        if ev is not None:
+            ev[1].record(stream)
+        binding.dendsn_lif_backward(cfg, x, gs, None, saved, gx, stream)
+        if ev is not None:
+            ev[2].record(stream)
+
+    for _ in range(warmup):
+        step()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    torch.cuda.synchronize()
+    for i in range(steps):
+        step(ev[i])
+    torch.cuda.synchronize()
+    fwd = statistics.mean(e[0].elapsed_time(e[1]) for e in ev)
+    bwd = statistics.mean(e[1].elapsed_time(e[2]) for e in ev)
+    ms = fwd + bwd
+    sx = x.element_size()
+    nbytes = T * B * N * 5 * sx            # fwd: x + S; bwd: x + gS + gX
+    return {"T": T, "B": B, "N": N, "x_dtype": dtype, "ms_per_step": ms, "forward_ms": fwd,
+            "backward_ms": bwd, "value": T * B * N / (ms / 1e3), "unit": UNIT,
+            "algorithmic_bytes_per_step": nbytes, "gbs": nbytes / (ms / 1e3) / 1e9}
+
+
 def run_ours(args):
     import torch
     import torch.distributed as dist
@@ -425,6 +464,21 @@ def run_ours(args):
         rate, sample, _, dt = oracle_sample_rate(w, cpu_inputs_from(w, inp), args.cpu_seconds)
         cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": sample + f", {dt:.1f} s", "host_cpus": os.cpu_count()}
+    lif = None
+    if not args.no_lif:
+        # the paper compares DendSN with LIF layers (Results, efficiency paragraph): here a
+        # LIF layer with the same neurons (one current each), and one fed the same input
+        # tensor (N*K point neurons)
+        steps_l = max(3, min(args.steps, 50))
+        same_n = time_lif(w.T, w.B, w.N, w.dtype, steps_l, 3, stream)
+        same_x = time_lif(w.T, w.B, w.N * w.K, w.dtype, steps_l, 3, stream)
+        for d in (same_n, same_x):
+            d["frac_of_measured"] = d["gbs"] / peak
+        lif = {"same_neurons": same_n, "same_input": same_x,
+               "dendsn_over_lif_same_neurons": value / world / same_n["value"],
+               "dendsn_over_lif_same_input": same_x["ms_per_step"] / step_ms,
+               "note": "layer-level ratios of fwd+bwd throughput; the paper's 0.92 is for "
+                       "whole networks (Tiny ImageNet VGG, Triton kernels)"}
     x_bytes = x.numel() * x.element_size()
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -447,6 +501,7 @@ def run_ours(args):
         "e2e": e2e,
         "gpu_launches": n_launch,
         "cpu_baseline": cpu,
+        "lif_baseline": lif,
     }
     print(json.dumps(line), flush=True)
     if world > 1:

@@ -145,6 +145,26 @@ dendsn_status dendsn_backward(const dendsn_config *cfg, const void *x, const flo
                               float *grad_kappa, void *scratch, void *stream);
 
 /*
+ * dendsn_backward for a soma whose decay beta is learnable (the PLIF soma the paper cites
+ * alongside LIF, read as Eq. methods-lif-reset-charge with beta a parameter). Same
+ * arguments and outputs as dendsn_backward, plus
+ *   grad_beta  [C] float32, OVERWRITTEN: dL/dbeta summed over time, samples and the
+ *              neurons of each channel, where dV^s[t+1]/dbeta = (1 - S[t]) V^s[t] (hard
+ *              reset) or V^s[t] - theta S[t] (soft). The gradient of the layer's single
+ *              beta is the sum of the C entries (parameterisations such as
+ *              beta = sigmoid(w) are applied by the caller).
+ * Runs a separate build of the backward kernel that also accumulates dL/dbeta (one more
+ * fused multiply-add per step); dendsn_backward does not pay for it.
+ */
+dendsn_status dendsn_backward_plif(const dendsn_config *cfg, const void *x, const float *alpha,
+                                   const float *xi, const float *zeta, const float *kappa,
+                                   const uint8_t *mask, const void *grad_spikes,
+                                   const float *grad_v, const void *saved, void *grad_x,
+                                   float *grad_alpha, float *grad_xi, float *grad_zeta,
+                                   float *grad_kappa, float *grad_beta, void *scratch,
+                                   void *stream);
+
+/*
  * Same computation and outputs as dendsn_backward, without the caller's scratch buffer:
  * for callers that cannot allocate device memory for it, such as a C host that only
  * receives device pointers for the layer's tensors, or a runtime whose device memory is
@@ -169,6 +189,39 @@ dendsn_status dendsn_backward_noalloc(const dendsn_config *cfg, const void *x,
                                       const void *saved, void *grad_x, float *grad_alpha,
                                       float *grad_xi, float *grad_zeta, float *grad_kappa,
                                       void *stream);
+
+/*
+ * Point-neuron LIF layer: the baseline neuron the paper compares the DendSN layer's speed
+ * with (Results, efficiency paragraph). It is the DendSN soma driven directly by one input
+ * current per neuron (Eq. methods-lif-reset-charge with X[t] in place of Z[t],
+ * Eq. methods-lif-fire; soft reset as above), trained with the same arctan surrogate
+ * (Eq. methods-sg). Same conventions as the DendSN entry points (device pointers, async
+ * on `stream`, host-side validation, dendsn_last_error()).
+ *   x, grad_x, spikes, grad_spikes   [T, B, N]  dtype x_dtype, naturally aligned
+ *   v_out, grad_v                    [T, B, N]  float32, 4-byte aligned; may be NULL
+ *   saved   checkpoints (V at the end of every 8 steps), saved_bytes of 16-byte aligned
+ *           device memory; needed (non-NULL) only when saved_bytes > 0, i.e. T > 8
+ * Tensors whose neuron count B*N is a multiple of 4 and whose pointers are aligned to 4
+ * elements (16 bytes for the float32 ones) take the vectorised kernels.
+ */
+typedef struct {
+    int32_t T, B, N;        /* time steps, samples, neurons per sample */
+    int32_t x_dtype;        /* dendsn_dtype of x, spikes, grad_spikes, grad_x */
+    int32_t reset;          /* dendsn_reset */
+    float theta, beta;      /* threshold, somatic decay (0 <= beta < 1) */
+    int32_t detach_reset;   /* 1: no gradient through the reset term */
+} dendsn_lif_config;
+
+dendsn_status dendsn_lif_workspace_size(const dendsn_lif_config *cfg, size_t *saved_bytes);
+
+/* Fused T-step LIF forward: writes spikes (and V if v_out), and the checkpoints to saved. */
+dendsn_status dendsn_lif_forward(const dendsn_lif_config *cfg, const void *x, void *spikes,
+                                 float *v_out, void *saved, void *stream);
+
+/* Fused reverse-time LIF backward: dL/dX from dL/dS (and dL/dV if grad_v), recomputing V. */
+dendsn_status dendsn_lif_backward(const dendsn_lif_config *cfg, const void *x,
+                                  const void *grad_spikes, const float *grad_v,
+                                  const void *saved, void *grad_x, void *stream);
 
 /* Static description of a status code. */
 const char *dendsn_status_string(dendsn_status status);

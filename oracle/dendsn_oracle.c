@@ -228,6 +228,8 @@ int oracle_forward(const oracle_cfg *cfg, const double *x, const int32_t *chan,
  *   gx [T][M][K]: dL/dX (overwritten).
  *   galpha, gxi [C][K], gzeta, gkappa [C][Kb]: summed over every neuron of a
  *   channel and every step (overwritten).
+ *   dvs [T][M] or NULL: dL/dV^s[t] (a diagnostic output: the tests derive from it
+ *   how strongly fp32 rounding of each branch's direction can show in grad_x).
  *   gbeta [C] or NULL: dL/dbeta of the somatic decay, summed the same way, for a
  *   soma whose beta is learnable (the PLIF soma the paper cites, read as
  *   Eq. methods-lif-reset-charge with beta a parameter):
@@ -238,7 +240,7 @@ int oracle_backward(const oracle_cfg *cfg, const double *x, const int32_t *chan,
                     const int32_t *mrow, const double *alpha, const double *xi,
                     const double *zeta, const double *kappa, const uint8_t *mask,
                     const double *gs, const double *gv, double *gx, double *galpha,
-                    double *gxi, double *gzeta, double *gkappa, double *gbeta)
+                    double *gxi, double *gzeta, double *gkappa, double *gbeta, double *dvs)
 {
     if (cfg == NULL || cfg->K <= 0 || cfg->G <= 0 || cfg->K % cfg->G != 0 || cfg->T < 0)
         return -1;
@@ -297,6 +299,8 @@ int oracle_backward(const oracle_cfg *cfg, const double *x, const int32_t *chan,
             double dv = surrogate_deriv(vs[t] - cfg->theta) * ds + dvdv_next * dv_next;
             if (gv != NULL)
                 dv += gv[(int64_t)t * M + m];
+            if (dvs != NULL)
+                dvs[(int64_t)t * M + m] = dv;
             const double dz = dv;
             /* Branches. */
             const double *vd = vd_hist + (int64_t)(t + 1) * K;

@@ -69,7 +69,7 @@ def build(force: bool = False) -> str:
 
 def _configure(lib):
     P = ctypes.c_void_p
-    for name, nargs in (("oracle_forward", 11), ("oracle_backward", 17),
+    for name, nargs in (("oracle_forward", 11), ("oracle_backward", 18),
                         ("oracle_lif_forward", 4), ("oracle_lif_backward", 5)):
         fn = getattr(lib, name)
         fn.restype = ctypes.c_int
@@ -162,20 +162,25 @@ def forward(c: OracleConfig, x, chan, mrow, alpha, xi, zeta, kappa, mask=None):
     return s, v
 
 
-def backward(c: OracleConfig, x, chan, mrow, alpha, xi, zeta, kappa, mask, gs, gv=None):
+def backward(c: OracleConfig, x, chan, mrow, alpha, xi, zeta, kappa, mask, gs, gv=None,
+             want_dvs: bool = False):
     """Backward of M neurons. Returns dict gx [T,M,K], galpha, gxi [C,K], gzeta, gkappa [C,Kb],
-    gbeta [C] (dL/dbeta per channel; a layer-wide beta's gradient is the sum)."""
+    gbeta [C] (dL/dbeta per channel; a layer-wide beta's gradient is the sum), and with
+    want_dvs also dvs [T,M] = dL/dV^s[t]."""
     x, M, chan, mrow, p, mask = _prep(c, x, chan, mrow, alpha, xi, zeta, kappa, mask)
     gs = to_f64(gs).reshape(c.T, M)
     gv = None if gv is None else to_f64(gv).reshape(c.T, M)
     out = dict(gx=np.zeros((c.T, M, c.K)), galpha=np.zeros((c.C, c.K)),
                gxi=np.zeros((c.C, c.K)), gzeta=np.zeros((c.C, c.Kb)),
                gkappa=np.zeros((c.C, c.Kb)), gbeta=np.zeros(c.C))
+    if want_dvs:
+        out["dvs"] = np.zeros((c.T, M))
     cfg = _cfg(c, M)
     rc = _load().oracle_backward(ctypes.byref(cfg), _ptr(x), _ptr(chan), _ptr(mrow),
                                  *[_ptr(a) for a in p], _ptr(mask), _ptr(gs), _ptr(gv),
                                  _ptr(out["gx"]), _ptr(out["galpha"]), _ptr(out["gxi"]),
-                                 _ptr(out["gzeta"]), _ptr(out["gkappa"]), _ptr(out["gbeta"]))
+                                 _ptr(out["gzeta"]), _ptr(out["gkappa"]), _ptr(out["gbeta"]),
+                                 _ptr(out.get("dvs")))
     if rc != 0:
         raise RuntimeError("oracle_backward failed")
     return out
@@ -281,12 +286,14 @@ def forward_layer(w, inp, **over):
     return s.reshape(w.T, w.B, w.N), v.reshape(w.T, w.B, w.N)
 
 
-def backward_layer(w, inp, gs=None, **over):
+def backward_layer(w, inp, gs=None, want_dvs=False, **over):
     """Oracle backward of a whole workload `w`; gs overrides inp['gs']."""
     chan, mrow = layer_channels(w.B, w.N, w.C, w.inner, w.mask_per_neuron)
     x = layer_x(w, inp["x"])
     gs = inp["gs"] if gs is None else gs
     out = backward(_cfg_of(w, **over), x, chan, mrow, inp["alpha"], inp["xi"], inp["zeta"],
-                   inp["kappa"], inp.get("mask"), gs, inp.get("gv"))
+                   inp["kappa"], inp.get("mask"), gs, inp.get("gv"), want_dvs=want_dvs)
     out["gx"] = layer_gx(w, out["gx"])
+    if want_dvs:
+        out["dvs"] = out["dvs"].reshape(w.T, w.B, w.N)
     return out

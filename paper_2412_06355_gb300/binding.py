@@ -68,6 +68,21 @@ def config_of(w) -> dendsn_config:
                        w.residual, layout=w.layout)
 
 
+class dendsn_lif_config(ctypes.Structure):
+    """Mirror of the C struct dendsn_lif_config (the point-neuron LIF layer)."""
+    _fields_ = [("T", ctypes.c_int32), ("B", ctypes.c_int32), ("N", ctypes.c_int32),
+                ("x_dtype", ctypes.c_int32), ("reset", ctypes.c_int32),
+                ("theta", ctypes.c_float), ("beta", ctypes.c_float),
+                ("detach_reset", ctypes.c_int32)]
+
+
+def make_lif_config(T, B, N, dtype="f32", reset="hard", theta=1.0, beta=0.5,
+                    detach_reset=False) -> dendsn_lif_config:
+    return dendsn_lif_config(T, B, N, BF16 if dtype == "bf16" else F32,
+                             RESET_SOFT if reset == "soft" else RESET_HARD, float(theta),
+                             float(beta), int(detach_reset))
+
+
 _lib = None
 _lock = threading.Lock()
 
@@ -88,7 +103,15 @@ def load() -> ctypes.CDLL:
                                                   ctypes.POINTER(ctypes.c_size_t)]
             lib.dendsn_forward.argtypes = [cfgp] + [P] * 10
             lib.dendsn_backward.argtypes = [cfgp] + [P] * 16
-            for fn in (lib.dendsn_workspace_size, lib.dendsn_forward, lib.dendsn_backward):
+            lib.dendsn_backward_plif.argtypes = [cfgp] + [P] * 17
+            lib.dendsn_backward_plif.restype = ctypes.c_int
+            lcfgp = ctypes.POINTER(dendsn_lif_config)
+            lib.dendsn_lif_workspace_size.argtypes = [lcfgp, ctypes.POINTER(ctypes.c_size_t)]
+            lib.dendsn_lif_forward.argtypes = [lcfgp] + [P] * 5
+            lib.dendsn_lif_backward.argtypes = [lcfgp] + [P] * 6
+            for fn in (lib.dendsn_workspace_size, lib.dendsn_forward, lib.dendsn_backward,
+                       lib.dendsn_lif_workspace_size, lib.dendsn_lif_forward,
+                       lib.dendsn_lif_backward):
                 fn.restype = ctypes.c_int
             lib.dendsn_status_string.argtypes = [ctypes.c_int]
             lib.dendsn_status_string.restype = ctypes.c_char_p
@@ -143,7 +166,8 @@ def _need(cfg, **tensors):
              "v_out": T * B * N * 4, "grad_v": T * B * N * 4,
              "alpha": C * K * 4, "xi": C * K * 4, "grad_alpha": C * K * 4, "grad_xi": C * K * 4,
              "zeta": C * Kb * 4, "kappa": C * Kb * 4, "grad_zeta": C * Kb * 4,
-             "grad_kappa": C * Kb * 4, "mask": (N if cfg.mask_per_neuron else C) * Kb}
+             "grad_kappa": C * Kb * 4, "mask": (N if cfg.mask_per_neuron else C) * Kb,
+             "grad_beta": C * 4}
     sizes = None
     for name, t in tensors.items():
         if t is None:
@@ -181,6 +205,21 @@ def dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, s
         _stream(stream)))
 
 
+def dendsn_backward_plif(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved,
+                         grad_x, grad_alpha, grad_xi, grad_zeta, grad_kappa, grad_beta, scratch,
+                         stream=None):
+    """dendsn_backward plus grad_beta [C], the gradient of a learnable somatic decay."""
+    _need(cfg, x=x, alpha=alpha, xi=xi, zeta=zeta, kappa=kappa, mask=mask,
+          grad_spikes=grad_spikes, grad_v=grad_v, saved=saved, grad_x=grad_x,
+          grad_alpha=grad_alpha, grad_xi=grad_xi, grad_zeta=grad_zeta, grad_kappa=grad_kappa,
+          grad_beta=grad_beta, scratch=scratch)
+    _check("dendsn_backward_plif", load().dendsn_backward_plif(
+        ctypes.byref(cfg), _ptr(x), _ptr(alpha), _ptr(xi), _ptr(zeta), _ptr(kappa),
+        _ptr(mask), _ptr(grad_spikes), _ptr(grad_v), _ptr(saved), _ptr(grad_x),
+        _ptr(grad_alpha), _ptr(grad_xi), _ptr(grad_zeta), _ptr(grad_kappa), _ptr(grad_beta),
+        _ptr(scratch), _stream(stream)))
+
+
 _noalloc_ready = False
 
 
@@ -205,6 +244,64 @@ def dendsn_backward_noalloc(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, g
         ctypes.byref(cfg), _ptr(x), _ptr(alpha), _ptr(xi), _ptr(zeta), _ptr(kappa),
         _ptr(mask), _ptr(grad_spikes), _ptr(grad_v), _ptr(saved), _ptr(grad_x),
         _ptr(grad_alpha), _ptr(grad_xi), _ptr(grad_zeta), _ptr(grad_kappa), _stream(stream)))
+
+
+# ------------------------------------------------------------------ point-neuron LIF layer
+def dendsn_lif_workspace_size(cfg: dendsn_lif_config) -> int:
+    """saved_bytes of the LIF layer (checkpoints; 0 for T <= 8)."""
+    s = ctypes.c_size_t(0)
+    _check("dendsn_lif_workspace_size",
+           load().dendsn_lif_workspace_size(ctypes.byref(cfg), ctypes.byref(s)))
+    return int(s.value)
+
+
+def _lif_need(cfg, **tensors):
+    sx = 2 if cfg.x_dtype == BF16 else 4
+    n = cfg.T * cfg.B * cfg.N
+    for name, t in tensors.items():
+        if t is None:
+            continue
+        need = (dendsn_lif_workspace_size(cfg) if name == "saved" else
+                n * 4 if name in ("v_out", "grad_v") else n * sx)
+        have = t.numel() * t.element_size()
+        if have < need:
+            raise ValueError(f"{name}: {have} bytes, the config needs {need}")
+
+
+def dendsn_lif_forward(cfg, x, spikes, v_out=None, saved=None, stream=None):
+    _lif_need(cfg, x=x, spikes=spikes, v_out=v_out, saved=saved)
+    _check("dendsn_lif_forward", load().dendsn_lif_forward(
+        ctypes.byref(cfg), _ptr(x), _ptr(spikes), _ptr(v_out), _ptr(saved), _stream(stream)))
+
+
+def dendsn_lif_backward(cfg, x, grad_spikes, grad_v, saved, grad_x, stream=None):
+    _lif_need(cfg, x=x, grad_spikes=grad_spikes, grad_v=grad_v, saved=saved, grad_x=grad_x)
+    _check("dendsn_lif_backward", load().dendsn_lif_backward(
+        ctypes.byref(cfg), _ptr(x), _ptr(grad_spikes), _ptr(grad_v), _ptr(saved),
+        _ptr(grad_x), _stream(stream)))
+
+
+def lif_forward(cfg, x, want_v=False, saved=None, stream=None):
+    """Allocating LIF forward of x [T, B, N]. Returns (spikes, v or None)."""
+    if tuple(x.shape) != (cfg.T, cfg.B, cfg.N) or x.dtype != _xdtype(cfg):
+        raise ValueError(f"x must be {_xdtype(cfg)} [{cfg.T},{cfg.B},{cfg.N}]")
+    spikes = torch.empty_like(x)
+    v = torch.empty(x.shape, dtype=torch.float32, device=x.device) if want_v else None
+    dendsn_lif_forward(cfg, x, spikes, v, saved, stream)
+    return spikes, v
+
+
+def lif_backward(cfg, x, grad_spikes, grad_v=None, saved=None, stream=None):
+    """Allocating LIF backward. Returns dL/dX with x's shape and dtype."""
+    gx = torch.empty_like(x)
+    dendsn_lif_backward(cfg, x, grad_spikes, grad_v, saved, gx, stream)
+    return gx
+
+
+def lif_workspace(cfg, device=None):
+    """The LIF checkpoint buffer, or None when T <= 8."""
+    sb = dendsn_lif_workspace_size(cfg)
+    return torch.empty(sb, dtype=torch.uint8, device=device or torch.device("cuda")) if sb else None
 
 
 # ------------------------------------------------------------------ tensor-level helpers
@@ -252,7 +349,8 @@ def forward(cfg, x, alpha, xi, zeta, kappa, mask=None, want_v=False, saved=None,
 
 def backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v=None, saved=None,
              scratch=None, stream=None):
-    """Allocating backward. Returns dict gx, galpha, gxi, gzeta, gkappa."""
+    """Allocating backward. Returns dict gx, galpha, gxi, gzeta, gkappa, gbeta (the last the
+    gradient of a learnable somatic decay, per channel)."""
     _check_shapes(cfg, x, alpha, xi, zeta, kappa, mask)
     if scratch is None:
         _, scratch = workspace(cfg, x.device)
@@ -262,10 +360,11 @@ def backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v=None, sav
                galpha=torch.empty((C, K), dtype=torch.float32, device=dev),
                gxi=torch.empty((C, K), dtype=torch.float32, device=dev),
                gzeta=torch.empty((C, Kb), dtype=torch.float32, device=dev),
-               gkappa=torch.empty((C, Kb), dtype=torch.float32, device=dev))
-    dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved,
-                    out["gx"], out["galpha"], out["gxi"], out["gzeta"], out["gkappa"],
-                    scratch, stream)
+               gkappa=torch.empty((C, Kb), dtype=torch.float32, device=dev),
+               gbeta=torch.empty((C,), dtype=torch.float32, device=dev))
+    dendsn_backward_plif(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved,
+                         out["gx"], out["galpha"], out["gxi"], out["gzeta"], out["gkappa"],
+                         out["gbeta"], scratch, stream)
     return out
 
 

@@ -13,11 +13,11 @@
 
 namespace dendsn {
 
-// Sums the block partials of every channel in a fixed order and writes the four
-// parameter gradients. One thread per (channel, gradient slot).
+// Sums the block partials of every channel in a fixed order and writes the parameter
+// gradients (grad_beta only when requested). One thread per (channel, gradient slot).
 __global__ void param_grad_finalize_kernel(const FinArgs F) {
     const Geometry &g = F.g;
-    const int NP = 2 * g.K + 2 * g.Kb;
+    const int NP = 2 * g.K + 2 * g.Kb + 1;
     const int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (w >= (int64_t)g.C * NP) return;
     const int c = (int)(w / NP);
@@ -35,11 +35,12 @@ __global__ void param_grad_finalize_kernel(const FinArgs F) {
     if (q < g.K) F.g_alpha[(int64_t)c * g.K + q] = F.stateless ? 0.f : sum;
     else if (q < 2 * g.K) F.g_xi[(int64_t)c * g.K + (q - g.K)] = sum;
     else if (q < 2 * g.K + g.Kb) F.g_zeta[(int64_t)c * g.Kb + (q - 2 * g.K)] = sum;
-    else F.g_kappa[(int64_t)c * g.Kb + (q - 2 * g.K - g.Kb)] = sum;
+    else if (q < 2 * g.K + 2 * g.Kb) F.g_kappa[(int64_t)c * g.Kb + (q - 2 * g.K - g.Kb)] = sum;
+    else if (F.g_beta) F.g_beta[c] = sum;
 }
 
 cudaError_t launch_finalize(const FinArgs &a, cudaStream_t s) {
-    const int64_t n = (int64_t)a.g.C * (2 * a.g.K + 2 * a.g.Kb);
+    const int64_t n = (int64_t)a.g.C * (2 * a.g.K + 2 * a.g.Kb + 1);
     const int threads = 256;
     const int blocks = (int)((n + threads - 1) / threads);
     param_grad_finalize_kernel<<<blocks, threads, 0, s>>>(a);
@@ -168,7 +169,7 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) 
     pl->blocks_b = (int)bb;
     pl->sx = (c.x_dtype == DENDSN_BF16) ? 2 : 4;
     pl->layout = (c.K > 1) ? c.layout : 0;
-    const size_t NP = 2 * (size_t)c.K + 2 * (size_t)g.Kb;
+    const size_t NP = 2 * (size_t)c.K + 2 * (size_t)g.Kb + 1;     // + the beta slot
     pl->scratch_bytes = (size_t)bb * pl->gb.nch_max * NP * sizeof(float);
     pl->scratch_bytes = (pl->scratch_bytes + 15) / 16 * 16;
     pl->ck_vd_bytes = (size_t)g.n_ck * (size_t)BN * c.K * sizeof(float);
@@ -294,12 +295,16 @@ dendsn_status dendsn_forward(const dendsn_config *cfg, const void *x, const floa
     return DENDSN_OK;
 }
 
-dendsn_status dendsn_backward(const dendsn_config *cfg, const void *x, const float *alpha,
-                              const float *xi, const float *zeta, const float *kappa,
-                              const uint8_t *mask, const void *grad_spikes,
-                              const float *grad_v, const void *saved, void *grad_x,
-                              float *grad_alpha, float *grad_xi, float *grad_zeta,
-                              float *grad_kappa, void *scratch, void *stream) {
+}  // extern "C"
+
+namespace {
+
+dendsn_status backward_impl(const dendsn_config *cfg, const void *x, const float *alpha,
+                            const float *xi, const float *zeta, const float *kappa,
+                            const uint8_t *mask, const void *grad_spikes,
+                            const float *grad_v, const void *saved, void *grad_x,
+                            float *grad_alpha, float *grad_xi, float *grad_zeta,
+                            float *grad_kappa, float *grad_beta, void *scratch, void *stream) {
     Plan pl;
     dendsn_status st = make_plan(cfg, &pl, true);
     if (st != DENDSN_OK) return st;
@@ -337,6 +342,7 @@ dendsn_status dendsn_backward(const dendsn_config *cfg, const void *x, const flo
                                 : nullptr;
         a.gx = grad_x;
         a.partials = static_cast<float *>(scratch);
+        a.want_beta = grad_beta != nullptr;
         cudaError_t e = dispatch_backward(*cfg, pl.layout, pl.gb.L, a, pl.blocks_b, s);
         if (e != cudaSuccess)
             return fail(DENDSN_ERR_CUDA, "backward launch failed: %s", cudaGetErrorString(e));
@@ -349,12 +355,42 @@ dendsn_status dendsn_backward(const dendsn_config *cfg, const void *x, const flo
     f.g_xi = grad_xi;
     f.g_zeta = grad_zeta;
     f.g_kappa = grad_kappa;
+    f.g_beta = grad_beta;
     f.stateless = cfg->stateless;
     cudaError_t e = launch_finalize(f, s);
     if (e != cudaSuccess)
         return fail(DENDSN_ERR_CUDA, "finalize launch failed: %s", cudaGetErrorString(e));
     g_launches.fetch_add(1, std::memory_order_relaxed);
     return DENDSN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+dendsn_status dendsn_backward(const dendsn_config *cfg, const void *x, const float *alpha,
+                              const float *xi, const float *zeta, const float *kappa,
+                              const uint8_t *mask, const void *grad_spikes,
+                              const float *grad_v, const void *saved, void *grad_x,
+                              float *grad_alpha, float *grad_xi, float *grad_zeta,
+                              float *grad_kappa, void *scratch, void *stream) {
+    return backward_impl(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved,
+                         grad_x, grad_alpha, grad_xi, grad_zeta, grad_kappa, nullptr, scratch,
+                         stream);
+}
+
+dendsn_status dendsn_backward_plif(const dendsn_config *cfg, const void *x, const float *alpha,
+                                   const float *xi, const float *zeta, const float *kappa,
+                                   const uint8_t *mask, const void *grad_spikes,
+                                   const float *grad_v, const void *saved, void *grad_x,
+                                   float *grad_alpha, float *grad_xi, float *grad_zeta,
+                                   float *grad_kappa, float *grad_beta, void *scratch,
+                                   void *stream) {
+    if (!grad_beta) return fail(DENDSN_ERR_INVALID_ARG, "grad_beta is NULL");
+    if (!aligned(grad_beta, 4)) return fail(DENDSN_ERR_MISALIGNED, "grad_beta must be 4-byte aligned");
+    return backward_impl(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved,
+                         grad_x, grad_alpha, grad_xi, grad_zeta, grad_kappa, grad_beta, scratch,
+                         stream);
 }
 
 const char *dendsn_status_string(dendsn_status status) {
@@ -435,3 +471,118 @@ extern "C" dendsn_status dendsn_backward_noalloc(
     return dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved,
                            grad_x, grad_alpha, grad_xi, grad_zeta, grad_kappa, scratch, stream);
 }
+
+// ------------------------------------------------------------------ point-neuron LIF layer
+namespace {
+
+struct LifPlan {
+    int64_t M;
+    int n_ck;          // checkpoints (T > 8 only)
+    int sx;
+};
+
+dendsn_status make_lif_plan(const dendsn_lif_config *cfg, LifPlan *pl) {
+    if (cfg == nullptr) return fail(DENDSN_ERR_INVALID_ARG, "cfg is NULL");
+    const dendsn_lif_config &c = *cfg;
+    if (c.T < 0 || c.B < 0 || c.N < 0)
+        return fail(DENDSN_ERR_INVALID_ARG, "negative size (T=%d B=%d N=%d)", c.T, c.B, c.N);
+    if (c.x_dtype != DENDSN_F32 && c.x_dtype != DENDSN_BF16)
+        return fail(DENDSN_ERR_INVALID_ARG, "bad x_dtype %d", c.x_dtype);
+    if ((c.reset != 0 && c.reset != 1) || (c.detach_reset != 0 && c.detach_reset != 1))
+        return fail(DENDSN_ERR_INVALID_ARG, "enum/flag field out of range");
+    if (!std::isfinite(c.theta) || !std::isfinite(c.beta))
+        return fail(DENDSN_ERR_INVALID_ARG, "theta and beta must be finite");
+    pl->M = (int64_t)c.B * c.N;
+    pl->n_ck = c.T > 8 ? (c.T + 7) / 8 - 1 : 0;
+    pl->sx = c.x_dtype == DENDSN_BF16 ? 2 : 4;
+    if ((pl->M + 3) / 4 > (int64_t)INT32_MAX * 256) return fail(DENDSN_ERR_UNSUPPORTED, "too many neurons");
+    return DENDSN_OK;
+}
+
+template <int XT>
+cudaError_t lif_dispatch(bool fwd, bool vec, const LifArgs &a, cudaStream_t s) {
+    if (fwd) return vec ? launch_lif_forward<XT, 4>(a, s) : launch_lif_forward<XT, 1>(a, s);
+    return vec ? launch_lif_backward<XT, 4>(a, s) : launch_lif_backward<XT, 1>(a, s);
+}
+
+}  // namespace
+
+extern "C" {
+
+dendsn_status dendsn_lif_workspace_size(const dendsn_lif_config *cfg, size_t *saved_bytes) {
+    LifPlan pl;
+    dendsn_status st = make_lif_plan(cfg, &pl);
+    if (st != DENDSN_OK) return st;
+    if (saved_bytes) *saved_bytes = ((size_t)pl.n_ck * pl.M * 4 + 15) / 16 * 16;
+    return DENDSN_OK;
+}
+
+dendsn_status dendsn_lif_forward(const dendsn_lif_config *cfg, const void *x, void *spikes,
+                                 float *v_out, void *saved, void *stream) {
+    LifPlan pl;
+    dendsn_status st = make_lif_plan(cfg, &pl);
+    if (st != DENDSN_OK) return st;
+    if (pl.M == 0 || cfg->T == 0) return DENDSN_OK;
+    if (!x || !spikes) return fail(DENDSN_ERR_INVALID_ARG, "x or spikes is NULL");
+    if (!aligned(x, pl.sx) || !aligned(spikes, pl.sx) || (v_out && !aligned(v_out, 4)))
+        return fail(DENDSN_ERR_MISALIGNED, "x, spikes or v_out misaligned");
+    if (saved && !aligned(saved, 16)) return fail(DENDSN_ERR_MISALIGNED, "saved must be 16-byte aligned");
+    const bool vec = pl.M % 4 == 0 && aligned(x, 4 * pl.sx) && aligned(spikes, 4 * pl.sx) &&
+                     (!v_out || aligned(v_out, 16));
+    LifArgs a{};
+    a.M = pl.M;
+    a.T = cfg->T;
+    a.theta = cfg->theta;
+    a.beta = cfg->beta;
+    a.soft = cfg->reset == DENDSN_RESET_SOFT;
+    a.detach_reset = cfg->detach_reset;
+    a.x = x;
+    a.spikes = spikes;
+    a.v_out = v_out;
+    a.ck = (saved && pl.n_ck > 0) ? static_cast<float *>(saved) : nullptr;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cfg->x_dtype == DENDSN_BF16 ? lif_dispatch<1>(true, vec, a, s)
+                                                : lif_dispatch<0>(true, vec, a, s);
+    if (e != cudaSuccess) return fail(DENDSN_ERR_CUDA, "LIF forward launch failed: %s", cudaGetErrorString(e));
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    return DENDSN_OK;
+}
+
+dendsn_status dendsn_lif_backward(const dendsn_lif_config *cfg, const void *x,
+                                  const void *grad_spikes, const float *grad_v,
+                                  const void *saved, void *grad_x, void *stream) {
+    LifPlan pl;
+    dendsn_status st = make_lif_plan(cfg, &pl);
+    if (st != DENDSN_OK) return st;
+    if (pl.M == 0 || cfg->T == 0) return DENDSN_OK;
+    if (!x || !grad_spikes || !grad_x) return fail(DENDSN_ERR_INVALID_ARG, "x, grad_spikes or grad_x is NULL");
+    if (!aligned(x, pl.sx) || !aligned(grad_spikes, pl.sx) || !aligned(grad_x, pl.sx) ||
+        (grad_v && !aligned(grad_v, 4)))
+        return fail(DENDSN_ERR_MISALIGNED, "x, grad_spikes, grad_x or grad_v misaligned");
+    if (pl.n_ck > 0 && !saved)
+        return fail(DENDSN_ERR_INVALID_ARG, "T=%d needs the forward's saved checkpoints", cfg->T);
+    if (saved && !aligned(saved, 16)) return fail(DENDSN_ERR_MISALIGNED, "saved must be 16-byte aligned");
+    const bool vec = pl.M % 4 == 0 && aligned(x, 4 * pl.sx) && aligned(grad_spikes, 4 * pl.sx) &&
+                     aligned(grad_x, 4 * pl.sx) && (!grad_v || aligned(grad_v, 16));
+    LifArgs a{};
+    a.M = pl.M;
+    a.T = cfg->T;
+    a.theta = cfg->theta;
+    a.beta = cfg->beta;
+    a.soft = cfg->reset == DENDSN_RESET_SOFT;
+    a.detach_reset = cfg->detach_reset;
+    a.x = x;
+    a.ck = pl.n_ck > 0 ? static_cast<float *>(const_cast<void *>(saved)) : nullptr;
+    a.gs = grad_spikes;
+    a.gv = grad_v;
+    a.gx = grad_x;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cfg->x_dtype == DENDSN_BF16 ? lif_dispatch<1>(false, vec, a, s)
+                                                : lif_dispatch<0>(false, vec, a, s);
+    if (e != cudaSuccess) return fail(DENDSN_ERR_CUDA, "LIF backward launch failed: %s", cudaGetErrorString(e));
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    return DENDSN_OK;
+}
+
+}  // extern "C"
+

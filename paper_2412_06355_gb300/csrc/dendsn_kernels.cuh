@@ -920,7 +920,9 @@ dendsn_forward_kernel(const FwdArgs A) {
 template <int KT, int G>
 constexpr int acc_count() { return 2 * KT + 2 * (KT / G); }
 
-template <int K, int G, int PSI, typename XT, int L, int LAYOUT>
+// BETA: also accumulate dL/dbeta (a learnable somatic decay); a separate instance because
+// even one more live accumulator slows the register-history path measurably.
+template <int K, int G, int PSI, typename XT, int L, int LAYOUT, bool BETA>
 __global__ void __launch_bounds__(bwd_threads(bwd_lane_compartments(K, G, xt_code<XT>(), L)),
                                   bwd_threads(bwd_lane_compartments(K, G, xt_code<XT>(), L)) == 128 ? 3 : 2)
 dendsn_backward_kernel(const BwdArgs A) {
@@ -1003,6 +1005,7 @@ dendsn_backward_kernel(const BwdArgs A) {
 
     typename AR::Acc acc;
     AR::acc_zero(acc);
+    float gbeta = 0.f;                // dL/dbeta (PLIF soma): sum of dL/dV^s[t+1] * leak[t]
 
     XRaw xb[BASYNC ? 1 : H];          // register ring: x of the next H steps to recompute
     typename S1::Raw gsb[L];          // grad_spikes of the current chunk
@@ -1156,6 +1159,11 @@ dendsn_backward_kernel(const BwdArgs A) {
                         vdp = (tt > 0) ? vdh[SHIST ? 0 : (tt > 0 ? tt - 1 : 0)] : vd0;
                     }
                     const bool st = vs >= P.theta;
+                    if constexpr (BETA) {
+                        // dV[t+1]/dbeta: (1 - S[t]) V[t] (hard) or V[t] - theta S[t] (soft)
+                        const float leak = st ? (P.soft ? __fsub_rn(vs, P.theta) : 0.f) : vs;
+                        gbeta = __fmaf_rn(dvn, leak, gbeta);
+                    }
                     const float dvds = __fmaf_rn(kv, vs, cs);               // dV[t+1]/dS[t]
                     const float dvdv = st ? b_spike : P.beta;               // dV[t+1]/dV[t]
                     const float ds = __fmaf_rn(dvds, dvn, gs_t);                          // dL/dS[t]
@@ -1179,15 +1187,18 @@ dendsn_backward_kernel(const BwdArgs A) {
     }
 
     // ---- parameter-gradient partials: per channel, fixed summation order
-    float v[NA];
+    // (slot NA: beta, counted once per neuron, by its first lane)
+    constexpr int NA1 = NA + 1;
+    float v[NA1];
     AR::acc_export(acc, v);
+    v[NA] = (BETA && pos.sub == 0) ? gbeta : 0.f;
 #pragma unroll
-    for (int a = 0; a < NA; ++a)
+    for (int a = 0; a < NA1; ++a)
         if (!pos.active || (a < KT && P.stateless)) v[a] = 0.f;
     // stage 1: within a warp, columns of one channel come in aligned runs of g.seg
     for (int d = 1; d < g.seg; d <<= 1) {
 #pragma unroll
-        for (int a = 0; a < NA; ++a)
+        for (int a = 0; a < NA1; ++a)
             v[a] = __fadd_rn(v[a], __shfl_xor_sync(0xffffffffu, v[a], d * LPN));
     }
     // stage 2: run leaders meet in shared memory; red[a][tid] (reuses the history space)
@@ -1195,20 +1206,21 @@ dendsn_backward_kernel(const BwdArgs A) {
     if constexpr (BASYNC) cp_async_wait<0>();
     __syncthreads();
 #pragma unroll
-    for (int a = 0; a < NA; ++a) red[a * NT + threadIdx.x] = v[a];
+    for (int a = 0; a < NA1; ++a) red[a * NT + threadIdx.x] = v[a];
     __syncthreads();
     const int ct = blockIdx.x % g.nCT;
     const int p0 = ct * g.TXn;
     const int p1 = min(p0 + g.TXn, g.P);            // exclusive
     const int c_lo = p0 / g.inner;
     const int nch = (p1 - 1) / g.inner - c_lo + 1;
-    const int NP = 2 * g.K + 2 * g.Kb;              // per-channel gradient vector
+    const int NP = 2 * g.K + 2 * g.Kb + 1;          // per-channel gradient vector
     float *out = A.partials + (int64_t)blockIdx.x * g.nch_max * NP;
-    const int items = nch * LPN * NA;
+    const int items = nch * LPN * NA1;
     for (int w = threadIdx.x; w < items; w += NT) {
-        const int a = w % NA;
-        const int sub = (w / NA) % LPN;
-        const int lc = w / (NA * LPN);
+        const int a = w % NA1;
+        const int sub = (w / NA1) % LPN;
+        const int lc = w / (NA1 * LPN);
+        if (a == NA && sub > 0) continue;          // beta: one lane per neuron
         const int c = c_lo + lc;
         const int cx_lo = max(c * g.inner, p0) - p0;
         const int cx_hi = min((c + 1) * g.inner, p1) - p0;
@@ -1220,7 +1232,8 @@ dendsn_backward_kernel(const BwdArgs A) {
         if (a < KT) slot = sub * KT + a;                                        // alpha
         else if (a < 2 * KT) slot = g.K + sub * KT + (a - KT);                  // xi
         else if (a < 2 * KT + KTb) slot = 2 * g.K + sub * KTb + (a - 2 * KT);   // zeta
-        else slot = 2 * g.K + g.Kb + sub * KTb + (a - 2 * KT - KTb);            // kappa
+        else if (a < NA) slot = 2 * g.K + g.Kb + sub * KTb + (a - 2 * KT - KTb); // kappa
+        else slot = NP - 1;                                                     // beta
         out[lc * NP + slot] = sum;
     }
 }
@@ -1252,16 +1265,22 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
     using T = typename XType<XT>::type;
     constexpr int KT = bwd_lane_compartments(K, G, XT, L);
     constexpr int NT = bwd_threads(KT);
-    const size_t red = sizeof(float) * acc_count<KT, G>() * NT;
+    const size_t red = sizeof(float) * (acc_count<KT, G>() + 1) * NT;
     constexpr bool shist = (L > 4) || KT >= 8;
     const size_t hist = shist ? sizeof(float) * (KT + 1) * L * NT : 0;
     using XI = XIO<T, KT, LAYOUT>;
     constexpr size_t xraw = sizeof(typename XI::Raw);
     const size_t ring = (DENDSN_BWD_ASYNC && shist && XI::kAsync) ? xraw * kBwdDepth * NT : 0;
     const size_t smem = red > hist + ring ? red : hist + ring;
-    cudaError_t e = allow_smem(dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT>, smem);
-    if (e != cudaSuccess) return e;
-    dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT><<<blocks, NT, smem, s>>>(a);
+    if (a.want_beta) {
+        cudaError_t e = allow_smem(dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, true>, smem);
+        if (e != cudaSuccess) return e;
+        dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, true><<<blocks, NT, smem, s>>>(a);
+    } else {
+        cudaError_t e = allow_smem(dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, false>, smem);
+        if (e != cudaSuccess) return e;
+        dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, false><<<blocks, NT, smem, s>>>(a);
+    }
     return cudaGetLastError();
 }
 

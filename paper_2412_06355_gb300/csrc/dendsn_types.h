@@ -69,13 +69,15 @@ struct BwdArgs {
     const float *ck_vd;
     const float *ck_vs;
     void *gx;
-    float *partials;   // [nCT * nRG][nch_max][NP], NP = 2K + 2Kb
+    float *partials;   // [nCT * nRG][nch_max][NP], NP = 2K + 2Kb + 1 (alpha, xi, zeta, kappa, beta)
+    int32_t want_beta; // accumulate the beta slot (else it stays zero)
 };
 
 struct FinArgs {
     Geometry g;
     const float *partials;
     float *g_alpha, *g_xi, *g_zeta, *g_kappa;
+    float *g_beta;     // [C] or null
     int32_t stateless;
 };
 
@@ -86,6 +88,28 @@ cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s);
 template <int K, int G, int PSI, int XT, int L, int LAYOUT>
 cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s);
 cudaError_t launch_finalize(const FinArgs &a, cudaStream_t s);
+
+// Point-neuron LIF layer: x, spikes, gs, gx are [T, M] in the x dtype; v_out and gv
+// [T, M] float32; ck [(T + 7) / 8 - 1, M] float32 somatic potentials at the ends of
+// the 8-step chunks (T > 4 only).
+struct LifArgs {
+    int64_t M;         // neurons
+    int32_t T;
+    float theta, beta;
+    int32_t soft, detach_reset;
+    const void *x;
+    void *spikes;
+    float *v_out;      // or null
+    float *ck;         // forward: written when not null; backward: read
+    const void *gs;
+    const float *gv;   // or null
+    void *gx;
+};
+
+// XT: 0 = float, 1 = bfloat16; VEC: neurons per thread (4 needs M % 4 == 0 and
+// 4-element-aligned tensors, else 1). Defined in lif_kernels.cu.
+template <int XT, int VEC> cudaError_t launch_lif_forward(const LifArgs &a, cudaStream_t s);
+template <int XT, int VEC> cudaError_t launch_lif_backward(const LifArgs &a, cudaStream_t s);
 
 }  // namespace dendsn
 

@@ -1,0 +1,11 @@
+// Explicit instantiations of the fused DendSN kernels (the backward with 8-step chunks): x dtype bfloat16,
+// psi = identity, compartments-innermost layout.
+// One translation unit per (dtype, psi, layout, part) so the library builds in parallel.
+#include "dendsn_kernels.cuh"
+
+namespace dendsn {
+#define DENDSN_INST(K, G) \
+    template cudaError_t launch_backward<K, G, 0, 1, 8, 0>(const BwdArgs &, int, cudaStream_t);
+DENDSN_KG_LIST(DENDSN_INST)
+#undef DENDSN_INST
+}  // namespace dendsn

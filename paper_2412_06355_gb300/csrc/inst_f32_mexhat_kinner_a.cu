@@ -1,0 +1,12 @@
+// Explicit instantiations of the fused DendSN kernels (forward and the backward with 4-step chunks): x dtype float32,
+// psi = Mexican hat, compartments-innermost layout.
+// One translation unit per (dtype, psi, layout, part) so the library builds in parallel.
+#include "dendsn_kernels.cuh"
+
+namespace dendsn {
+#define DENDSN_INST(K, G) \
+    template cudaError_t launch_forward<K, G, 1, 0, 0>(const FwdArgs &, int, cudaStream_t);     \
+    template cudaError_t launch_backward<K, G, 1, 0, 4, 0>(const BwdArgs &, int, cudaStream_t);
+DENDSN_KG_LIST(DENDSN_INST)
+#undef DENDSN_INST
+}  // namespace dendsn

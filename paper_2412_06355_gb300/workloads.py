@@ -89,9 +89,10 @@ class Workload:
         return dataclasses.replace(self, **kw)
 
 
-# The five layer shapes: a tiny case, a conv layer, a deeper bf16 conv layer, a
-# long-horizon event-stream layer with sparse input, and a transformer-token layer
-# with per-neuron branch gating.
+# The layer shapes: a tiny case, a conv layer (also in the paper's (C_o, P, H, W) layout
+# with two compartments per branch), a deeper bf16 conv layer, a long-horizon
+# event-stream layer with sparse input, a transformer-token layer with per-neuron branch
+# gating, and two T = 2048 cases.
 WORKLOADS = {
     "tiny": Workload("tiny", T=4, B=2, N=64, K=4, G=1, C=64, inner=1, dtype="f32",
                      psi="mh", reset="hard", seed=0),
@@ -108,6 +109,15 @@ WORKLOADS = {
     "token_dbg": Workload("token_dbg", T=4, B=64, N=196 * 384, K=8, G=1, C=384, inner=1,
                           dtype="f32", psi="mh", reset="hard", mask_p=0.5,
                           mask_per_neuron=True, seed=4),
+    # long horizon: the L5PC fitting setting (one neuron with P = 4 compartments on
+    # B = 2 branches, T = 2048, batch 16, beta = 0.95; Methods "Details of L5PC
+    # approximation" and the hyperparameter table), and the same horizon on a layer
+    "l5pc": Workload("l5pc", T=2048, B=16, N=1, K=4, G=2, C=1, inner=1, dtype="f32",
+                     psi="mh", reset="hard", beta=0.95, x_mean=0.1, x_std=0.5,
+                     x_density=0.3, seed=6),
+    "long_t": Workload("long_t", T=2048, B=16, N=4096, K=4, G=2, C=4, inner=1024,
+                       dtype="f32", psi="mh", reset="hard", beta=0.95, x_mean=0.1,
+                       x_std=0.5, x_density=0.3, seed=7),
 }
 
 
@@ -146,6 +156,22 @@ def make_inputs(w: Workload, device: str = "cpu", with_gv: bool = False) -> dict
     gs = torch.randn((T, B, N), generator=g, **f32).to(torch_dtype(w))
     gv = torch.randn((T, B, N), generator=g, **f32) if with_gv else None
     return dict(x=x, alpha=alpha, xi=xi, zeta=zeta, kappa=kappa, mask=mask, gs=gs, gv=gv)
+
+
+def make_lif_inputs(T: int, B: int, N: int, dtype: str = "f32", seed: int = 0,
+                    device: str = "cpu", with_gv: bool = False, x_mean: float = 0.5,
+                    x_std: float = 1.0) -> dict:
+    """Inputs of the point-neuron LIF layer: x ~ N(x_mean, x_std) [T, B, N] (one current
+    per neuron), gs ~ N(0, 1) [T, B, N] in the layer dtype, gv ~ N(0, 1) float32.
+    Draw order x, gs, gv from one generator."""
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    f32 = dict(dtype=torch.float32, device=device)
+    dt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    x = torch.randn((T, B, N), generator=g, **f32).mul_(x_std).add_(x_mean).to(dt)
+    gs = torch.randn((T, B, N), generator=g, **f32).to(dt)
+    gv = torch.randn((T, B, N), generator=g, **f32) if with_gv else None
+    return dict(x=x, gs=gs, gv=gv)
 
 
 def to_paper_layout(x: torch.Tensor, inner: int) -> torch.Tensor:

@@ -48,12 +48,15 @@ def test_library_exports_every_declared_symbol(lib):
         assert hasattr(lib, name)
 
 
-def test_config_layout_matches_c():
-    fields = [f[0] for f in binding.dendsn_config._fields_]
+@pytest.mark.parametrize("struct", [binding.dendsn_config, binding.dendsn_lif_config],
+                         ids=lambda s: s.__name__)
+def test_config_layout_matches_c(struct):
+    name = struct.__name__
+    fields = [f[0] for f in struct._fields_]
     prog = "#include <stdio.h>\n#include <stddef.h>\n#include \"dendsn.h\"\nint main(void){\n"
-    prog += 'printf("%zu\\n", sizeof(dendsn_config));\n'
+    prog += f'printf("%zu\\n", sizeof({name}));\n'
     for f in fields:
-        prog += f'printf("%zu\\n", offsetof(dendsn_config, {f}));\n'
+        prog += f'printf("%zu\\n", offsetof({name}, {f}));\n'
     prog += "return 0;}\n"
     with tempfile.TemporaryDirectory() as d:
         c = os.path.join(d, "t.c")
@@ -61,9 +64,9 @@ def test_config_layout_matches_c():
         open(c, "w").write(prog)
         subprocess.check_call(["gcc", "-std=c99", "-I", os.path.join(ROOT, "include"), c, "-o", exe])
         vals = [int(v) for v in subprocess.check_output([exe]).split()]
-    assert vals[0] == ctypes.sizeof(binding.dendsn_config)
+    assert vals[0] == ctypes.sizeof(struct)
     for f, off in zip(fields, vals[1:]):
-        assert getattr(binding.dendsn_config, f).offset == off, f
+        assert getattr(struct, f).offset == off, f
 
 
 def status_of(fn, *args):
@@ -155,6 +158,25 @@ def test_binding_refuses_undersized_tensors(lib):
     with pytest.raises(ValueError, match="scratch"):
         binding.dendsn_backward(cfg, x, *p, None, torch.zeros(4, 2, 64), None, None,
                                 torch.zeros_like(x), *p, torch.zeros(1))
+
+
+def test_lif_validation_and_workspace(lib):
+    mk = binding.make_lif_config
+    assert binding.dendsn_lif_workspace_size(mk(T=8, B=2, N=10)) == 0
+    assert binding.dendsn_lif_workspace_size(mk(T=9, B=2, N=10)) == 80      # 1 x 20 x 4 B
+    assert binding.dendsn_lif_workspace_size(mk(T=64, B=3, N=7)) == (7 * 21 * 4 + 15) // 16 * 16
+    for bad in (dict(T=-1), dict(reset=2), dict(x_dtype=5), dict(theta=float("inf"))):
+        cfg = mk(T=4, B=2, N=10)
+        for k, v in bad.items():
+            setattr(cfg, k, v)
+        assert status_of(binding.dendsn_lif_workspace_size, cfg) == 1, bad
+    P = ctypes.c_void_p
+    cfg = mk(T=4, B=1, N=64)
+    assert lib.dendsn_lif_forward(ctypes.byref(cfg), None, P(4096), None, None, None) == 1
+    assert lib.dendsn_lif_forward(ctypes.byref(cfg), P(4098), P(4096), None, None, None) == 3
+    cfg = mk(T=20, B=1, N=64)       # needs checkpoints
+    assert lib.dendsn_lif_backward(ctypes.byref(cfg), P(4096), P(4096), None, None, P(4096),
+                                   None) == 1
 
 
 def test_status_strings(lib):

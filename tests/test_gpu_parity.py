@@ -19,7 +19,8 @@ from paper_2412_06355_gb300 import binding, workloads
 from paper_2412_06355_gb300.workloads import WORKLOADS, scaled
 
 from parity import (BF16_ATOL_REL, BF16_RTOL, G_ATOL_REL, G_RTOL, V_ATOL, V_RTOL,
-                    assert_close, check_layer, first_ambiguous_step, to_dev)
+                    assert_close, check_layer, direction_rounding_allowance,
+                    first_ambiguous_step, gx_atol_rel, to_dev)
 
 pytestmark = pytest.mark.gpu
 
@@ -40,6 +41,8 @@ SCALED = {
     "token_dbg": scaled(WORKLOADS["token_dbg"], B=2),
     "conv_paper_p4b2": scaled(WORKLOADS["conv_paper_p4b2"], B=2),
     "deepconv_bf16_paper": scaled(WORKLOADS["deepconv_bf16"], B=2).with_(layout="paper"),
+    "l5pc": WORKLOADS["l5pc"],
+    "long_t": WORKLOADS["long_t"].with_(B=1, N=1024, C=1),
 }
 
 
@@ -89,7 +92,7 @@ def test_paper_layout_is_bitwise_the_kinner_layer(K, G, T, dtype):
     (s, v, g), (sp, vp, gp) = outs
     assert torch.equal(s, sp) and torch.equal(v, vp)
     assert torch.equal(g["gx"], workloads.from_paper_layout(gp["gx"], w.N, w.K, w.inner))
-    for k in ("galpha", "gxi", "gzeta", "gkappa"):
+    for k in ("galpha", "gxi", "gzeta", "gkappa", "gbeta"):
         assert torch.equal(g[k], gp[k]), k
 
 
@@ -152,7 +155,7 @@ def test_empty_shapes():
                              inp["gs"], None)
         torch.cuda.synchronize()
         assert s.numel() == 0
-        for k in ("galpha", "gxi", "gzeta", "gkappa"):
+        for k in ("galpha", "gxi", "gzeta", "gkappa", "gbeta"):
             assert torch.count_nonzero(g[k]).item() == 0
 
 
@@ -269,10 +272,14 @@ def test_full_size_sampled(name, kw):
     sm = t_idx < first[None]
     assert np.array_equal(got_s[sm], s_o[sm])
 
-    ref = oracle.backward(ocfg, xs, chan, mrow, *prm, mask, gs_sample[:, bt, nt].cpu())
-    rt, ar = (BF16_RTOL, BF16_ATOL_REL) if w.dtype == "bf16" else (G_RTOL, G_ATOL_REL)
-    assert_close("grad_x", got_gx, ref["gx"], rt, ar)
-    for k in ("galpha", "gxi", "gzeta", "gkappa"):
+    ref = oracle.backward(ocfg, xs, chan, mrow, *prm, mask, gs_sample[:, bt, nt].cpu(),
+                          want_dvs=True)
+    extra = direction_rounding_allowance(w, oracle.to_f64(xs), chan, mrow, *prm, mask,
+                                         ref["dvs"])
+    rt, ar = ((BF16_RTOL, BF16_ATOL_REL) if w.dtype == "bf16"
+              else (G_RTOL, gx_atol_rel(w, inp["alpha"])))
+    assert_close("grad_x", got_gx, ref["gx"], rt, ar, atol_abs=extra)
+    for k in ("galpha", "gxi", "gzeta", "gkappa", "gbeta"):
         assert_close(k, oracle.to_f64(g[k]), ref[k], G_RTOL, G_ATOL_REL)
     # every non-sampled neuron received zero upstream gradient: its grad_x is zero
     gx = g["gx"]
