@@ -158,28 +158,41 @@ template <int XT> struct XType;
 template <> struct XType<0> { using type = float; };
 template <> struct XType<1> { using type = __nv_bfloat16; };
 
-// Mask bits of KTb branches of one lane, as 1.0f / 0.0f.
+// Mask bits of KTb branches of one lane: fetched raw (one or two 32-bit loads, so a
+// row's mask can be requested a row ahead of its use), then unpacked to 1.0f / 0.0f.
+template <int KTb> struct MaskRaw { using T = typename std::conditional<KTb == 8, uint2, uint32_t>::type; };
+
 template <int KTb>
-__device__ __forceinline__ void load_mask(const uint8_t *m, float (&mk)[KTb]) {
+__device__ __forceinline__ typename MaskRaw<KTb>::T fetch_mask(const uint8_t *m) {
     if constexpr (KTb == 8) {
-        const uint32_t q0 = __ldg(reinterpret_cast<const unsigned int *>(m));
-        const uint32_t q1 = __ldg(reinterpret_cast<const unsigned int *>(m) + 1);
+        return make_uint2(__ldg(reinterpret_cast<const unsigned int *>(m)),
+                          __ldg(reinterpret_cast<const unsigned int *>(m) + 1));
+    } else if constexpr (KTb == 4) {
+        return __ldg(reinterpret_cast<const unsigned int *>(m));
+    } else if constexpr (KTb == 2) {
+        return __ldg(reinterpret_cast<const unsigned short *>(m));
+    } else {
+        return __ldg(m);
+    }
+}
+
+template <int KTb>
+__device__ __forceinline__ void unpack_mask(const typename MaskRaw<KTb>::T &q, float (&mk)[KTb]) {
+    if constexpr (KTb == 8) {
 #pragma unroll
         for (int b = 0; b < 4; ++b) {
-            mk[b] = ((q0 >> (8 * b)) & 0xffu) ? 1.f : 0.f;
-            mk[4 + b] = ((q1 >> (8 * b)) & 0xffu) ? 1.f : 0.f;
+            mk[b] = ((q.x >> (8 * b)) & 0xffu) ? 1.f : 0.f;
+            mk[4 + b] = ((q.y >> (8 * b)) & 0xffu) ? 1.f : 0.f;
         }
-    } else if constexpr (KTb == 4) {
-        const uint32_t q = __ldg(reinterpret_cast<const unsigned int *>(m));
-#pragma unroll
-        for (int b = 0; b < 4; ++b) mk[b] = ((q >> (8 * b)) & 0xffu) ? 1.f : 0.f;
-    } else if constexpr (KTb == 2) {
-        const uint32_t q = __ldg(reinterpret_cast<const unsigned short *>(m));
-        mk[0] = (q & 0xffu) ? 1.f : 0.f;
-        mk[1] = (q >> 8) ? 1.f : 0.f;
     } else {
-        mk[0] = __ldg(m) ? 1.f : 0.f;
+#pragma unroll
+        for (int b = 0; b < KTb; ++b) mk[b] = ((q >> (8 * b)) & 0xffu) ? 1.f : 0.f;
     }
+}
+
+template <int KTb>
+__device__ __forceinline__ void load_mask(const uint8_t *m, float (&mk)[KTb]) {
+    unpack_mask<KTb>(fetch_mask<KTb>(m), mk);
 }
 
 // ---------------------------------------------------------------- arithmetic
@@ -242,10 +255,16 @@ __device__ __forceinline__ void load_param_arrays(const Params &P, const Geometr
 
 // kappa * m and m for the neuron n of a per-neuron mask (mask_mode 2).
 template <int KTb>
-__device__ __forceinline__ void load_neuron_mask(const Params &P, const Geometry &g, int64_t n,
-                                                 int chan, int sub, float (&km)[KTb],
-                                                 float (&mk)[KTb]) {
-    load_mask<KTb>(P.mask + n * g.Kb + sub * KTb, mk);
+__device__ __forceinline__ typename MaskRaw<KTb>::T fetch_neuron_mask(const Params &P, const Geometry &g,
+                                                                      int64_t n, int sub) {
+    return fetch_mask<KTb>(P.mask + n * g.Kb + sub * KTb);
+}
+
+template <int KTb>
+__device__ __forceinline__ void apply_neuron_mask(const Params &P, const Geometry &g,
+                                                  const typename MaskRaw<KTb>::T &raw, int chan,
+                                                  int sub, float (&km)[KTb], float (&mk)[KTb]) {
+    unpack_mask<KTb>(raw, mk);
 #pragma unroll
     for (int b = 0; b < KTb; ++b)
         km[b] = __fmul_rn(__ldg(P.kappa + (int64_t)chan * g.Kb + sub * KTb + b), mk[b]);
@@ -273,9 +292,13 @@ struct PairArith {
             lp.mk[m] = make_float2(mk[2 * m], mk[2 * m + 1]);
         }
     }
-    static __device__ __forceinline__ void neuron_mask(const Params &P, const Geometry &g, int64_t n, int chan, int sub, LP &lp) {
+    using MRaw = typename MaskRaw<KTb>::T;
+    static __device__ __forceinline__ MRaw fetch_neuron_mask(const Params &P, const Geometry &g, int64_t n, int sub) {
+        return dendsn::fetch_neuron_mask<KT>(P, g, n, sub);
+    }
+    static __device__ __forceinline__ void neuron_mask(const Params &P, const Geometry &g, const MRaw &raw, int chan, int sub, LP &lp) {
         float km[KT], mk[KT];
-        load_neuron_mask<KT>(P, g, n, chan, sub, km, mk);
+        apply_neuron_mask<KT>(P, g, raw, chan, sub, km, mk);
 #pragma unroll
         for (int m = 0; m < N2; ++m) {
             lp.km[m] = make_float2(km[2 * m], km[2 * m + 1]);
@@ -428,8 +451,12 @@ struct ScalarArith {
     static __device__ __forceinline__ void load(const Params &P, const Geometry &g, int chan, int sub, LP &lp) {
         load_param_arrays<KT, G>(P, g, chan, sub, lp.a, lp.nxi, lp.iz, lp.km, lp.mk);
     }
-    static __device__ __forceinline__ void neuron_mask(const Params &P, const Geometry &g, int64_t n, int chan, int sub, LP &lp) {
-        load_neuron_mask<KTb>(P, g, n, chan, sub, lp.km, lp.mk);
+    using MRaw = typename MaskRaw<KTb>::T;
+    static __device__ __forceinline__ MRaw fetch_neuron_mask(const Params &P, const Geometry &g, int64_t n, int sub) {
+        return dendsn::fetch_neuron_mask<KTb>(P, g, n, sub);
+    }
+    static __device__ __forceinline__ void neuron_mask(const Params &P, const Geometry &g, const MRaw &raw, int chan, int sub, LP &lp) {
+        apply_neuron_mask<KTb>(P, g, raw, chan, sub, lp.km, lp.mk);
     }
     static __device__ __forceinline__ void zero(St &s) {
 #pragma unroll
@@ -555,6 +582,30 @@ template <int KT, int G, int PSI, typename XT>
 using Arith = typename std::conditional<(G == 1 && KT % 2 == 0),
                                         PairArith<KT, PSI, std::is_same<XT, float>::value>,
                                         ScalarArith<KT, G, PSI>>::type;
+
+// Per-neuron branch masks (mask_mode 2) of a thread's rows, each fetched one row ahead of
+// its use so the row start does not wait on the load. n: the neuron (within a sample) of
+// the next row; step: the thread's row stride in neurons, modulo N.
+template <typename AR>
+struct MaskAhead {
+    typename AR::MRaw next;
+    int n, step;
+    __device__ __forceinline__ void init(const Params &P, const Geometry &g, int64_t j0,
+                                         int64_t jstep, int sub, int nrows) {
+        n = (int)(j0 % g.N);
+        step = (int)(jstep % g.N);
+        if (P.mask_mode == 2 && nrows > 0) next = AR::fetch_neuron_mask(P, g, n, sub);
+    }
+    // applies the current row's mask, then requests the next row's (if `more`)
+    __device__ __forceinline__ void advance(const Params &P, const Geometry &g, int chan, int sub,
+                                            bool more, typename AR::LP &lp) {
+        if (P.mask_mode != 2) return;
+        AR::neuron_mask(P, g, next, chan, sub, lp);
+        n += step;
+        if (n >= g.N) n -= g.N;
+        if (more) next = AR::fetch_neuron_mask(P, g, n, sub);
+    }
+};
 
 // Sum of the LPN lanes' shares (xor butterfly: every lane gets the same bits).
 template <int LPN>
@@ -790,8 +841,10 @@ dendsn_forward_kernel(const FwdArgs A) {
             const XT *xr = xrow;
             XT *sr = srow;
             float *vr = vrow;
+            MaskAhead<AR> mask;
+            mask.init(P, g, j0, jstep, pos.sub, pos.nrows);
             for (int i = 0; i < pos.nrows; ++i) {
-                if (P.mask_mode == 2) AR::neuron_mask(P, g, j % g.N, pos.chan, pos.sub, lp);
+                mask.advance(P, g, pos.chan, pos.sub, i + 1 < pos.nrows, lp);
                 typename AR::St vd;
                 AR::zero(vd);
                 float v = 0.f;
@@ -866,8 +919,10 @@ dendsn_forward_kernel(const FwdArgs A) {
         }
     }
     int64_t j = j0;
+    MaskAhead<AR> mask;
+    mask.init(P, g, j0, jstep, pos.sub, pos.nrows);
     for (int i = 0; i < pos.nrows; ++i) {
-        if (P.mask_mode == 2) AR::neuron_mask(P, g, j % g.N, pos.chan, pos.sub, lp);
+        mask.advance(P, g, pos.chan, pos.sub, i + 1 < pos.nrows, lp);
         typename AR::St vd;
         AR::zero(vd);
         float v = 0.f;
@@ -1034,8 +1089,10 @@ dendsn_backward_kernel(const BwdArgs A) {
     }
 
     int64_t j = j0;
+    MaskAhead<AR> mask;
+    mask.init(P, g, j0, jstep, pos.sub, pos.nrows);
     for (int i = 0; i < pos.nrows; ++i) {
-        if (P.mask_mode == 2) AR::neuron_mask(P, g, j % g.N, pos.chan, pos.sub, lp);
+        mask.advance(P, g, pos.chan, pos.sub, i + 1 < pos.nrows, lp);
         typename AR::St Ad;           // dL/dV^d[t+1], carried backwards
         AR::zero(Ad);
         float dvn = 0.f;              // dL/dV^s[t+1]

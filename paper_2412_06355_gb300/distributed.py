@@ -33,6 +33,12 @@ def param_grad_buffer(C: int, K: int, Kb: int, device=None) -> Tuple[torch.Tenso
                   "gkappa": gk.view(C, Kb)}
 
 
+def split_param_grads(flat: torch.Tensor, C: int, K: int, Kb: int):
+    """(galpha, gxi, gzeta, gkappa) views of one flat parameter-gradient row."""
+    ga, gxi, gz, gk = torch.split(flat, [C * K, C * K, C * Kb, C * Kb])
+    return ga.view(C, K), gxi.view(C, K), gz.view(C, Kb), gk.view(C, Kb)
+
+
 def sum_param_grads(flat: torch.Tensor, group=None) -> torch.Tensor:
     """Sums the parameter-gradient buffer over the ranks of `group` in place."""
     if dist.is_available() and dist.is_initialized() and dist.get_world_size(group) > 1:
