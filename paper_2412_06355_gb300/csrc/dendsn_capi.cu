@@ -168,7 +168,7 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) 
     pl->blocks_f = (int)bf;
     pl->blocks_b = (int)bb;
     pl->sx = (c.x_dtype == DENDSN_BF16) ? 2 : 4;
-    pl->layout = (c.K > 1) ? c.layout : 0;
+    pl->layout = (c.K > 1 && c.inner > 1) ? c.layout : 0;   // otherwise the layouts coincide
     const size_t NP = 2 * (size_t)c.K + 2 * (size_t)g.Kb + 1;     // + the beta slot
     pl->scratch_bytes = (size_t)bb * pl->gb.nch_max * NP * sizeof(float);
     pl->scratch_bytes = (pl->scratch_bytes + 15) / 16 * 16;

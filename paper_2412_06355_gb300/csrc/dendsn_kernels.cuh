@@ -971,6 +971,130 @@ dendsn_forward_kernel(const FwdArgs A) {
     }
 }
 
+// Forward in the paper's (C_o, P, H, W) layout with the inputs staged per warp. Used when a
+// lane serves a whole neuron (K <= 8) and H*W and the column tile are multiples of 32: a
+// warp's 32 neurons are then 32 consecutive positions of one channel group, so compartment k
+// of all of them is one contiguous run of 32 elements. Each lane copies its share of the
+// warp's K runs with 16-byte cp.async into the slot [k][32 lanes] (one copy per lane per
+// step for 4 float32 compartments, as in the compartments-innermost layout) and reads back
+// its own neuron's K values. Ordering: every lane waits for its own copy groups, then
+// __syncwarp() makes all lanes' copies visible; a slot is refilled one step after it was
+// read, behind that same barrier, so kFwdDepth - 1 steps are in flight.
+template <int K, int G, int PSI, typename XT>
+__global__ void __launch_bounds__(fwd_threads(K), K >= 8 ? 2 : DENDSN_FWD_MINB)
+dendsn_forward_staged_kernel(const FwdArgs A) {
+    constexpr int NT = fwd_threads(K);
+    constexpr int KT = K;                        // one lane per neuron
+    constexpr int D = kFwdDepth;
+    constexpr int SX = (int)sizeof(XT);
+    constexpr int EPC = 16 / SX;                 // elements per 16-byte chunk
+    constexpr int CPK = 32 / EPC;                // chunks per compartment run of a warp
+    constexpr int NCH = K * CPK;                 // chunks per warp per step
+    constexpr int CPL = (NCH + 31) / 32;         // chunks per lane
+    using AR = Arith<KT, G, PSI, XT>;
+    const Geometry &g = A.g;
+    const Params &P = A.p;
+    const ThreadPos pos = thread_pos<1>(g);
+    // whole warps: rows are uniform per warp, and P % 32 == 0 makes activity uniform too
+    if (pos.nrows == 0 || !pos.active) return;
+    typename AR::LP lp;
+    AR::load(P, g, pos.chan, 0, lp);
+    const float inv_k = 1.f / (float)K;
+    const int T = g.T;
+    const int64_t sX = g.BN * K;
+    const int64_t BN = g.BN;
+    const int64_t j0 = pos.row0 * g.P + pos.p;
+    const int64_t jstep = (int64_t)pos.rstride * g.P;
+    const int64_t rX = jstep * K;
+    const int lane = threadIdx.x & 31;
+    // the warp's first neuron: 32-aligned position, so every chunk is 16-byte aligned
+    const XT *xw = static_cast<const XT *>(A.x) + lane_x_offset<1>(j0, 0, KT, K, g.inner) - lane;
+    XT *sp = static_cast<XT *>(A.spikes) + j0;
+    float *vp = A.v_out ? A.v_out + j0 : nullptr;
+    const bool write_ck = (A.ck_vd != nullptr) && g.n_ck > 0;
+    const bool residual = P.residual != 0;
+
+    extern __shared__ float4 fwd_smem[];
+    constexpr int kSlot = NT * K;                // elements of one slot (all warps)
+    XT *wring = reinterpret_cast<XT *>(fwd_smem) + (threadIdx.x >> 5) * (32 * K);
+    int64_t src[CPL];
+    int dst[CPL];
+#pragma unroll
+    for (int m = 0; m < CPL; ++m) {
+        const int c = lane + 32 * m;
+        const int kc = c / CPK, pc = c % CPK;
+        src[m] = (int64_t)kc * g.inner + pc * EPC;
+        dst[m] = kc * 32 + pc * EPC;
+    }
+    auto fetch = [&](int slot, const XT *base) {
+#pragma unroll
+        for (int m = 0; m < CPL; ++m)
+            if (lane + 32 * m < NCH) cp_async<16>(wring + slot * kSlot + dst[m], base + src[m], 0.f);
+    };
+    // fetch walker over this thread's (row, step) sequence
+    const XT *ip = xw;
+    int it = 0, ir = 0;
+    const int64_t row_jump = rX - (int64_t)T * sX;
+    auto walk = [&]() {
+        ip += sX;
+        if (++it == T) { it = 0; ++ir; ip += row_jump; }
+    };
+#pragma unroll
+    for (int k = 0; k < D - 1; ++k) {
+        if (ir < pos.nrows) fetch(k, ip);
+        cp_async_commit();
+        walk();
+    }
+    int slot = 0;
+    int64_t j = j0;
+    MaskAhead<AR> mask;
+    mask.init(P, g, j0, jstep, 0, pos.nrows);
+    for (int i = 0; i < pos.nrows; ++i) {
+        mask.advance(P, g, pos.chan, 0, i + 1 < pos.nrows, lp);
+        typename AR::St vd;
+        AR::zero(vd);
+        float v = 0.f;
+        bool s = false;
+        XT *spt = sp;
+        float *vpt = vp;
+        for (int t = 0; t < T; ++t) {
+            cp_async_wait<D - 2>();
+            __syncwarp();
+            // refill the slot every lane read in the previous step
+            if (ir < pos.nrows) fetch(slot == 0 ? D - 1 : slot - 1, ip);
+            cp_async_commit();
+            walk();
+            float xv[KT];
+#pragma unroll
+            for (int k = 0; k < KT; ++k) {
+                if constexpr (SX == 4) xv[k] = reinterpret_cast<const float *>(wring)[slot * kSlot + k * 32 + lane];
+                else xv[k] = bf16_lo(reinterpret_cast<const unsigned short *>(wring)[slot * kSlot + k * 32 + lane]);
+            }
+            const float z = soma_input<AR, KT, 1>(lp, vd, xv, residual, inv_k);
+            v = soma_charge(z, v, s, P);
+            s = v >= P.theta;                    // Eq. methods-lif-fire
+            Scalar<XT>::store_spike(spt, s);
+            if (vpt) {
+                __stcs(vpt, v);
+                vpt += BN;
+            }
+            spt += BN;
+            if (write_ck && ((t + 1) & (g.L - 1)) == 0 && t + 1 < T) {
+                const int ck = (t + 1) / g.L - 1;
+                float vda[KT];
+                AR::to_array(vd, vda);
+                Vec<float, KT>::store(A.ck_vd + ((int64_t)ck * BN + j) * K, vda);
+                __stcs(A.ck_vs + (int64_t)ck * BN + j, v);
+            }
+            slot = (slot == D - 1) ? 0 : slot + 1;
+        }
+        sp += jstep;
+        if (vp) vp += jstep;
+        j += jstep;
+    }
+    cp_async_wait<0>();
+}
+
 // ---------------------------------------------------------------- backward
 template <int KT, int G>
 constexpr int acc_count() { return 2 * KT + 2 * (KT / G); }
@@ -1310,6 +1434,16 @@ cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s) {
     using XI = XIO<T, KT, LAYOUT>;
     constexpr size_t raw = sizeof(typename XI::Raw);
     constexpr int NT = fwd_threads(K);
+    if constexpr (LAYOUT == 1 && K >= 2 && K <= 8 && DENDSN_FWD_ASYNC) {
+        // the paper layout with warps of 32 consecutive positions: staged per warp
+        if (a.g.inner % 32 == 0 && a.g.TXn % 32 == 0) {
+            const size_t smem = (size_t)kFwdDepth * NT * K * sizeof(T);
+            cudaError_t e = allow_smem(dendsn_forward_staged_kernel<K, G, PSI, T>, smem);
+            if (e != cudaSuccess) return e;
+            dendsn_forward_staged_kernel<K, G, PSI, T><<<blocks, NT, smem, s>>>(a);
+            return cudaGetLastError();
+        }
+    }
     const size_t smem = (DENDSN_FWD_ASYNC && XI::kAsync) ? raw * kFwdDepth * NT : 0;
     cudaError_t e = allow_smem(dendsn_forward_kernel<K, G, PSI, T, LAYOUT>, smem);
     if (e != cudaSuccess) return e;

@@ -70,12 +70,13 @@ def test_every_compiled_kg(K, G, layout):
     check_layer(w)
 
 
+@pytest.mark.parametrize("inner", [40, 64])      # 64: the forward stages inputs per warp
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("K,G,T", [(2, 2, 3), (4, 2, 4), (4, 1, 12), (8, 1, 4), (8, 2, 9),
                                    (16, 4, 5)])
-def test_paper_layout_is_bitwise_the_kinner_layer(K, G, T, dtype):
+def test_paper_layout_is_bitwise_the_kinner_layer(K, G, T, dtype, inner):
     """Only the addresses differ between the layouts: every output must be bit-identical."""
-    w = workloads.Workload("lay", T=T, B=3, N=4 * 2 * 40, K=K, G=G, C=4, inner=40,
+    w = workloads.Workload("lay", T=T, B=3, N=4 * 2 * inner, K=K, G=G, C=4, inner=inner,
                            dtype=dtype, psi="mh", reset="hard", mask_p=0.7, seed=21)
     wp = w.with_(layout="paper")
     outs = []
