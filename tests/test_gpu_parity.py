@@ -233,9 +233,16 @@ FULL = [(n, {}) for n in WORKLOADS] + [
 ]
 
 
-@pytest.mark.parametrize("name,kw", FULL, ids=[n + "".join(f"-{k}" for k in kw) for n, kw in FULL])
+# element offsets beyond 2^31: T * B * N * K = 64 * 65 * 131072 * 4 = 2.18e9 (x alone 8.7 GB)
+BIG = workloads.Workload("offsets_beyond_int32", T=64, B=65, N=131072, K=4, G=1, C=128,
+                         inner=1024, dtype="f32", psi="mh", reset="hard", seed=41)
+
+
+@pytest.mark.parametrize("name,kw", FULL + [("offsets_beyond_int32", {})],
+                         ids=[n + "".join(f"-{k}" for k in kw) for n, kw in FULL] +
+                         ["offsets_beyond_int32"])
 def test_full_size_sampled(name, kw):
-    w = WORKLOADS[name].with_(**kw)
+    w = (BIG if name == BIG.name else WORKLOADS[name]).with_(**kw)
     cfg = binding.config_of(w)
     inp = workloads.make_inputs(w, "cuda")          # full size, generated on the device
     b_idx, n_idx = sample_neurons(w, 3000, seed=w.seed)
