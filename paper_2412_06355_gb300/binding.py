@@ -348,9 +348,10 @@ def forward(cfg, x, alpha, xi, zeta, kappa, mask=None, want_v=False, saved=None,
 
 
 def backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v=None, saved=None,
-             scratch=None, stream=None):
-    """Allocating backward. Returns dict gx, galpha, gxi, gzeta, gkappa, gbeta (the last the
-    gradient of a learnable somatic decay, per channel)."""
+             scratch=None, stream=None, want_beta=False):
+    """Allocating backward. Returns dict gx, galpha, gxi, gzeta, gkappa, and with want_beta
+    also gbeta (the gradient of a learnable somatic decay, per channel; computed by the
+    separate dendsn_backward_plif kernel build)."""
     _check_shapes(cfg, x, alpha, xi, zeta, kappa, mask)
     if scratch is None:
         _, scratch = workspace(cfg, x.device)
@@ -360,29 +361,39 @@ def backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v=None, sav
                galpha=torch.empty((C, K), dtype=torch.float32, device=dev),
                gxi=torch.empty((C, K), dtype=torch.float32, device=dev),
                gzeta=torch.empty((C, Kb), dtype=torch.float32, device=dev),
-               gkappa=torch.empty((C, Kb), dtype=torch.float32, device=dev),
-               gbeta=torch.empty((C,), dtype=torch.float32, device=dev))
-    dendsn_backward_plif(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved,
-                         out["gx"], out["galpha"], out["gxi"], out["gzeta"], out["gkappa"],
-                         out["gbeta"], scratch, stream)
+               gkappa=torch.empty((C, Kb), dtype=torch.float32, device=dev))
+    grads = (out["gx"], out["galpha"], out["gxi"], out["gzeta"], out["gkappa"])
+    if want_beta:
+        out["gbeta"] = torch.empty((C,), dtype=torch.float32, device=dev)
+        dendsn_backward_plif(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved,
+                             *grads, out["gbeta"], scratch, stream)
+    else:
+        dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, grad_spikes, grad_v, saved,
+                        *grads, scratch, stream)
     return out
 
 
 class DendSNFunction(torch.autograd.Function):
-    """autograd wrapper: S = DendSN(X; alpha, xi, zeta, kappa) (Eq. dendsn).
+    """autograd wrapper: S = DendSN(X; alpha, xi, zeta, kappa[, beta]) (Eq. dendsn).
 
-    alpha may be a scalar tensor (the paper's layer-wide decay) or [C, K]; its
-    gradient is reduced to its own shape. The mask is a constant.
+    alpha may be a scalar tensor (the paper's layer-wide decay) or [C, K]; its gradient is
+    reduced to its own shape. The mask is a constant. beta: None (the somatic decay is
+    cfg.beta, a constant) or a 0-dim tensor, a learnable decay (PLIF soma); its value
+    replaces cfg.beta and its gradient is the sum of the per-channel dL/dbeta.
     """
 
     @staticmethod
-    def forward(ctx, x, alpha, xi, zeta, kappa, mask, cfg):
+    def forward(ctx, x, alpha, xi, zeta, kappa, mask, cfg, beta=None):
+        if beta is not None:
+            cfg = dendsn_config.from_buffer_copy(cfg)
+            cfg.beta = float(beta)
         a = alpha.expand(cfg.C, cfg.K).contiguous().float()
         saved, scratch = workspace(cfg, x.device)
         s, _ = forward(cfg, x.contiguous(), a, xi.contiguous(), zeta.contiguous(),
                        kappa.contiguous(), mask, saved=saved)
         ctx.cfg = cfg
         ctx.alpha_shape = alpha.shape
+        ctx.learn_beta = beta is not None
         ctx.ws = (saved, scratch)
         ctx.save_for_backward(x, a, xi, zeta, kappa, mask)
         return s
@@ -392,6 +403,7 @@ class DendSNFunction(torch.autograd.Function):
         x, a, xi, zeta, kappa, mask = ctx.saved_tensors
         saved, scratch = ctx.ws
         g = backward(ctx.cfg, x, a, xi, zeta, kappa, mask, gs.contiguous().to(x.dtype),
-                     None, saved, scratch)
+                     None, saved, scratch, want_beta=ctx.learn_beta)
         ga = g["galpha"].sum_to_size(ctx.alpha_shape)
-        return g["gx"], ga, g["gxi"], g["gzeta"], g["gkappa"], None, None
+        gb = g["gbeta"].sum() if ctx.learn_beta else None
+        return g["gx"], ga, g["gxi"], g["gzeta"], g["gkappa"], None, None, gb

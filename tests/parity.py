@@ -133,7 +133,12 @@ def run_gpu(w, inp_dev: dict, gs, gv, want_v=True):
                            inp_dev["zeta"], inp_dev["kappa"], inp_dev["mask"], want_v=want_v,
                            saved=saved)
     g = binding.backward(cfg, inp_dev["x"], inp_dev["alpha"], inp_dev["xi"], inp_dev["zeta"],
-                         inp_dev["kappa"], inp_dev["mask"], gs, gv, saved, scratch)
+                         inp_dev["kappa"], inp_dev["mask"], gs, gv, saved, scratch, want_beta=True)
+    # the plain backward (the kernel build without dL/dbeta) gives the same bits elsewhere
+    g0 = binding.backward(cfg, inp_dev["x"], inp_dev["alpha"], inp_dev["xi"], inp_dev["zeta"],
+                          inp_dev["kappa"], inp_dev["mask"], gs, gv, saved, scratch)
+    for k in g0:
+        assert torch.equal(g0[k], g[k]), f"{k} differs between the backward builds"
     # the production forward (no V^s output; checkpoints when T needs them) must give
     # the same spikes and the same checkpoints bit for bit
     saved2, _ = binding.workspace(cfg)

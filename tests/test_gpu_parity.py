@@ -87,7 +87,8 @@ def test_paper_layout_is_bitwise_the_kinner_layer(K, G, T, dtype, inner):
         s, v = binding.forward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"],
                                inp["kappa"], inp["mask"], want_v=True, saved=saved)
         g = binding.backward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"],
-                             inp["kappa"], inp["mask"], inp["gs"], inp["gv"], saved, scratch)
+                             inp["kappa"], inp["mask"], inp["gs"], inp["gv"], saved, scratch,
+                             want_beta=True)
         outs.append((s, v, g))
     torch.cuda.synchronize()
     (s, v, g), (sp, vp, gp) = outs
@@ -153,7 +154,7 @@ def test_empty_shapes():
         inp = to_dev(workloads.make_inputs(w, "cpu"))
         s, _ = binding.forward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"], None)
         g = binding.backward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"], None,
-                             inp["gs"], None)
+                             inp["gs"], None, want_beta=True)
         torch.cuda.synchronize()
         assert s.numel() == 0
         for k in ("galpha", "gxi", "gzeta", "gkappa", "gbeta"):
@@ -170,7 +171,8 @@ def test_backward_is_deterministic():
         binding.forward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"],
                         inp["mask"], saved=saved)
         outs.append(binding.backward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"],
-                                     inp["kappa"], inp["mask"], inp["gs"], None, saved, scratch))
+                                     inp["kappa"], inp["mask"], inp["gs"], None, saved, scratch,
+                                     want_beta=True))
     for k in outs[0]:
         assert torch.equal(outs[0][k], outs[1][k]), k
 
@@ -207,6 +209,30 @@ def test_autograd_function_layer_wide_alpha():
     assert torch.allclose(alpha.grad, ref["galpha"].sum(), rtol=1e-5, atol=1e-6)
     assert torch.equal(x.grad, ref["gx"])
     assert torch.equal(kappa.grad, ref["gkappa"])
+
+
+def test_autograd_function_learnable_beta():
+    """A learnable somatic decay (PLIF soma) through autograd: its gradient is the sum of the
+    per-channel dL/dbeta, checked against the float64 oracle."""
+    w = workloads.Workload("plif", T=6, B=2, N=128, K=4, G=2, C=4, inner=32, dtype="f32",
+                           psi="mh", reset="soft", beta=0.8, seed=23)
+    inp = workloads.make_inputs(w, "cpu")
+    dev = to_dev(inp)
+    cfg = binding.config_of(w.with_(beta=0.5))          # the tensor's value must win
+    beta = torch.tensor(0.8, device="cuda", requires_grad=True)
+    x = dev["x"].clone().requires_grad_(True)
+    s = binding.DendSNFunction.apply(x, dev["alpha"], dev["xi"], dev["zeta"], dev["kappa"],
+                                     None, cfg, beta)
+    s_o, v_o = oracle.forward_layer(w, inp)
+    amb = torch.from_numpy(first_ambiguous_step(v_o, w.theta) < w.T)
+    gs = inp["gs"].clone()
+    gs[:, amb] = 0
+    assert np.array_equal(oracle.to_f64(s)[:, ~amb.numpy()], s_o[:, ~amb.numpy()])
+    (s * gs.cuda()).sum().backward()
+    ref = oracle.backward_layer(w, inp, gs=gs)
+    assert_close("dL/dbeta", [beta.grad.item()], [ref["gbeta"].sum()], G_RTOL, G_ATOL_REL,
+                 atol_abs=1e-5 * float(np.sqrt(np.mean(ref["gbeta"] ** 2))))
+    assert_close("grad_x", oracle.to_f64(x.grad), ref["gx"], G_RTOL, G_ATOL_REL)
 
 
 # ------------------------------------------------------------------ full size, sampled
@@ -270,7 +296,7 @@ def test_full_size_sampled(name, kw):
     s, v = binding.forward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"],
                            inp["mask"], want_v=True, saved=saved)
     g = binding.backward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"], inp["kappa"],
-                         inp["mask"], gs_sample, None, saved, scratch)
+                         inp["mask"], gs_sample, None, saved, scratch, want_beta=True)
     torch.cuda.synchronize()
     got_s = oracle.to_f64(s[:, bt, nt])
     got_v = oracle.to_f64(v[:, bt, nt])
