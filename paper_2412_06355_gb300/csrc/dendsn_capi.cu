@@ -220,7 +220,7 @@ dendsn_status check_params(const float *alpha, const float *xi, const float *zet
         }                                                                               \
     }
 
-// layout: 0 compartments innermost, 1 the paper's layer layout (same as 0 when K = 1)
+// layout: 0 compartments innermost, 1 the paper's layer layout (0 when K = 1 or inner = 1: the same)
 cudaError_t dispatch_forward(const dendsn_config &cfg, int layout, const FwdArgs &a, int blocks,
                              cudaStream_t s) {
     DENDSN_KG_LIST(DENDSN_FWD_CASE)

@@ -7,8 +7,12 @@
 // TXn columns x TY row lanes; each neuron is served by LPN adjacent lanes of one
 // warp that own KT = K / LPN compartments each (16 bytes of fp32 input per step,
 // one 128-bit load). A thread walks up to R rows of its column, and each row's T
-// steps in order. Loads run a fixed number of steps ahead of use through a small
-// ring of registers, across chunk and row boundaries.
+// steps in order. Inputs are fetched a fixed number of steps ahead of use, across
+// chunk and row boundaries: through a per-thread ring of shared-memory slots filled
+// by cp.async (the forward; the backward of multi-chunk rows), or a ring of
+// registers (the backward of rows of at most 4 steps). In the paper's (C_o, P, H, W)
+// layout a lane's compartments are H*W apart; when H*W is a multiple of 32 the
+// forward stages each warp's inputs together (dendsn_forward_staged_kernel).
 //
 // Forward (Eqs. methods-compartment .. methods-lif-fire): V^d, V^s and S stay in
 // registers across all T steps; the HBM traffic per step is the K inputs read and
@@ -29,6 +33,9 @@
 // (__ffma2_rn and friends round each component exactly like __fmaf_rn), which
 // halves the floating-point instruction count; G > 1 uses a scalar engine.
 // Address arithmetic is pointer increments; 64-bit divisions happen once per thread.
+//
+// Waits. The kernels never spin: cp.async.wait_group waits on the thread's own copies,
+// __syncwarp / __syncthreads on threads that always reach them.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -775,8 +782,9 @@ __device__ __forceinline__ int64_t lane_x_offset(int64_t j, int sub, int KT, int
     return (j - s) * K + s + (int64_t)sub * KT * inner;
 }
 
-// x is prefetched kFwdBatch steps ahead of use (a ring of kFwdBatch registers);
-// checkpoints every g.L steps (g.L is a power of two and a multiple of the batch).
+// x is fetched kFwdDepth steps ahead of use through the cp.async ring (or, without it, a
+// ring of kFwdBatch registers); checkpoints every g.L steps (g.L is a power of two and a
+// multiple of the batch).
 // Lanes of 8 compartments: 3 blocks per SM for float32 (measured 2% faster), 2 for bf16
 // (whose unpacking spills under the tighter cap, 15% slower).
 template <int K, int G, int PSI, typename XT, int LAYOUT>
