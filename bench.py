@@ -43,6 +43,8 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--plif", action="store_true",
+                    help="learnable somatic decay: time dendsn_backward_plif (adds dL/dbeta)")
     ap.add_argument("--no-lif", action="store_true",
                     help="skip timing the point-neuron LIF layer baseline")
     ap.add_argument("--workload", default="conv")
@@ -365,6 +367,7 @@ def run_ours(args):
     gx = torch.empty_like(x)
     grads, views = distributed.param_grad_buffer(w.C, w.K, w.Kb, dev)
     ga, gxi, gz, gk = (views[k] for k in ("galpha", "gxi", "gzeta", "gkappa"))
+    gbeta = torch.empty(w.C, dtype=torch.float32, device=dev)     # --plif: dL/dbeta
     stream = torch.cuda.current_stream()
 
     def step(ev=None):
@@ -373,8 +376,12 @@ def run_ours(args):
         binding.dendsn_forward(cfg, x, alpha, xi, zeta, kappa, mask, spikes, None, saved, stream)
         if ev is not None:
             ev[1].record(stream)
-        binding.dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, gs, None, saved, gx,
-                                ga, gxi, gz, gk, scratch, stream)
+        if args.plif:
+            binding.dendsn_backward_plif(cfg, x, alpha, xi, zeta, kappa, mask, gs, None, saved,
+                                         gx, ga, gxi, gz, gk, gbeta, scratch, stream)
+        else:
+            binding.dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, gs, None, saved, gx,
+                                    ga, gxi, gz, gk, scratch, stream)
         if ev is not None:
             ev[2].record(stream)
         if world > 1:
@@ -541,10 +548,12 @@ def run_ours(args):
         "config": config_dict(w, {
             "l2": f"inputs larger than L2: x is {x_bytes / 2**20:.0f} MiB per step "
                   f"(L2 {L2_BYTES // 2**20} MiB), no flush",
-            "parallelism": f"dp{world}" if world > 1 else "single GPU"}),
+            "parallelism": f"dp{world}" if world > 1 else "single GPU",
+            "soma": "plif (learnable beta)" if args.plif else "lif"}),
         "roofline": {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peak,
                      "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
-                     "traffic": recorded_traffic(kname, w.name),
+                     # counters were taken on the plain backward build, not the dL/dbeta one
+                     "traffic": None if args.plif else recorded_traffic(kname, w.name),
                      "algorithmic_bytes_per_launch": kbytes, "avg_launch_ms": kms},
         "hbm": {"algorithmic_bytes_per_step": ab["total"],
                 "step_gbs": ab["total"] / (step_ms / 1e3) / 1e9,
