@@ -322,3 +322,49 @@ def test_full_size_sampled(name, kw):
     gx_abs = gx.abs().sum(dim=(0, 3))
     gx_abs[bt, nt] = 0
     assert torch.count_nonzero(gx_abs).item() == 0
+
+
+# ------------------------------------------------------------------ CUDA graphs
+def test_cuda_graph_capture_and_replay():
+    """A whole step (forward, backward, finalize) captured into a CUDA graph and replayed on
+    new inputs written into the captured buffers gives the eager calls' bits."""
+    w = workloads.Workload("graph", T=12, B=2, N=4 * 64, K=4, G=2, C=4, inner=64, dtype="f32",
+                           psi="mh", reset="hard", mask_p=0.5, seed=51)
+    cfg = binding.config_of(w)
+    inp = to_dev(workloads.make_inputs(w, "cpu"))
+    x, gs = inp["x"].clone(), inp["gs"].clone()
+    p = [inp[k] for k in ("alpha", "xi", "zeta", "kappa")]
+    saved, scratch = binding.workspace(cfg)
+    spikes = torch.empty((w.T, w.B, w.N), device="cuda")
+    gx = torch.empty_like(x)
+    grads = [torch.empty_like(t) for t in p]
+
+    def step(stream):
+        binding.dendsn_forward(cfg, x, *p, inp["mask"], spikes, None, saved, stream)
+        binding.dendsn_backward(cfg, x, *p, inp["mask"], gs, None, saved, gx, *grads, scratch,
+                                stream)
+
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        step(side)                                    # warm-up outside the capture
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step(torch.cuda.current_stream())
+    for seed in (52, 53):
+        new = workloads.make_inputs(w.with_(seed=seed), "cpu")
+        x.copy_(new["x"])
+        gs.copy_(new["gs"])
+        graph.replay()
+        torch.cuda.synchronize()
+        s_eager, _ = binding.forward(cfg, x, *p, inp["mask"], saved=binding.workspace(cfg)[0])
+        sv, sc = binding.workspace(cfg)
+        binding.forward(cfg, x, *p, inp["mask"], saved=sv)
+        g = binding.backward(cfg, x, *p, inp["mask"], gs, None, sv, sc)
+        torch.cuda.synchronize()
+        assert torch.equal(spikes, s_eager)
+        assert torch.equal(gx, g["gx"])
+        for got, k in zip(grads, ("galpha", "gxi", "gzeta", "gkappa")):
+            assert torch.equal(got, g[k]), k
