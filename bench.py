@@ -43,6 +43,8 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--graph", action="store_true",
+                    help="replay the forward and backward as captured CUDA graphs")
     ap.add_argument("--plif", action="store_true",
                     help="learnable somatic decay: time dendsn_backward_plif (adds dL/dbeta)")
     ap.add_argument("--no-lif", action="store_true",
@@ -370,18 +372,48 @@ def run_ours(args):
     gbeta = torch.empty(w.C, dtype=torch.float32, device=dev)     # --plif: dL/dbeta
     stream = torch.cuda.current_stream()
 
+    def fwd(strm):
+        binding.dendsn_forward(cfg, x, alpha, xi, zeta, kappa, mask, spikes, None, saved, strm)
+
+    def bwd(strm):
+        if args.plif:
+            binding.dendsn_backward_plif(cfg, x, alpha, xi, zeta, kappa, mask, gs, None, saved,
+                                         gx, ga, gxi, gz, gk, gbeta, scratch, strm)
+        else:
+            binding.dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, gs, None, saved, gx,
+                                    ga, gxi, gz, gk, scratch, strm)
+
+    # --graph: the forward and the backward each captured into a CUDA graph once, then
+    # replayed every step (no per-step host launch work; events stay between the replays)
+    launches_per_step = None
+    if args.graph:
+        if world > 1:
+            raise SystemExit("--graph times one GPU")
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):               # one eager step before capturing
+            fwd(side)
+            bwd(side)
+        stream.wait_stream(side)
+        torch.cuda.synchronize()
+        n0 = binding.launch_count()
+        graphs = []
+        for part in (fwd, bwd):
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr):
+                part(torch.cuda.current_stream())
+            graphs.append(gr)
+        launches_per_step = binding.launch_count() - n0
+        fwd = lambda strm: graphs[0].replay()     # noqa: E731  (replays on the current stream)
+        bwd = lambda strm: graphs[1].replay()     # noqa: E731
+
     def step(ev=None):
         if ev is not None:
             ev[0].record(stream)
-        binding.dendsn_forward(cfg, x, alpha, xi, zeta, kappa, mask, spikes, None, saved, stream)
+        fwd(stream)
         if ev is not None:
             ev[1].record(stream)
-        if args.plif:
-            binding.dendsn_backward_plif(cfg, x, alpha, xi, zeta, kappa, mask, gs, None, saved,
-                                         gx, ga, gxi, gz, gk, gbeta, scratch, stream)
-        else:
-            binding.dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, gs, None, saved, gx,
-                                    ga, gxi, gz, gk, scratch, stream)
+        bwd(stream)
         if ev is not None:
             ev[2].record(stream)
         if world > 1:
@@ -406,6 +438,8 @@ def run_ours(args):
     torch.cuda.synchronize()
     t1 = time.time()
     n_launch = binding.launch_count() - n_launch0
+    if launches_per_step is not None:               # replays launch without library calls
+        n_launch = launches_per_step * args.steps
     if world > 1:
         dist.barrier()
     ms = start.elapsed_time(end)
@@ -549,7 +583,8 @@ def run_ours(args):
             "l2": f"inputs larger than L2: x is {x_bytes / 2**20:.0f} MiB per step "
                   f"(L2 {L2_BYTES // 2**20} MiB), no flush",
             "parallelism": f"dp{world}" if world > 1 else "single GPU",
-            "soma": "plif (learnable beta)" if args.plif else "lif"}),
+            "soma": "plif (learnable beta)" if args.plif else "lif",
+            "launch": "cuda graph replay" if args.graph else "eager"}),
         "roofline": {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peak,
                      "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
                      # counters were taken on the plain backward build, not the dL/dbeta one
