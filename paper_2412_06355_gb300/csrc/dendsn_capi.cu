@@ -72,6 +72,7 @@ struct Plan {
     size_t saved_bytes, scratch_bytes, ck_vd_bytes;
     int sx;            // bytes per x element
     int layout;        // 0 compartments innermost, 1 the paper's layer layout
+    bool tp;           // the time-parallel kernels (one warp per neuron)
 };
 
 int sm_count() {
@@ -172,6 +173,14 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) 
     const size_t NP = 2 * (size_t)c.K + 2 * (size_t)g.Kb + 1;     // + the beta slot
     pl->scratch_bytes = (size_t)bb * pl->gb.nch_max * NP * sizeof(float);
     pl->scratch_bytes = (pl->scratch_bytes + 15) / 16 * 16;
+    // narrow layers with long horizons: one warp per neuron, time scanned in parallel
+    pl->tp = c.T >= kTpMinT && BN <= kTpMaxNeurons && tp_smem_bytes(c.T, c.K, true) <= kTpMaxSmem;
+    if (pl->tp) {
+        pl->gf.n_ck = pl->gb.n_ck = 0;                 // the backward recomputes from x alone
+        pl->scratch_bytes = ((size_t)BN * NP * sizeof(float) + 15) / 16 * 16;
+        pl->ck_vd_bytes = pl->saved_bytes = 0;
+        return DENDSN_OK;
+    }
     pl->ck_vd_bytes = (size_t)g.n_ck * (size_t)BN * c.K * sizeof(float);
     pl->saved_bytes = pl->ck_vd_bytes + (size_t)g.n_ck * (size_t)BN * sizeof(float);
     pl->saved_bytes = (pl->saved_bytes + 15) / 16 * 16;
@@ -251,6 +260,25 @@ cudaError_t dispatch_backward(const dendsn_config &cfg, int layout, int L, const
     return cudaErrorInvalidValue;
 }
 
+#define DENDSN_TP_FWD_CASE(KK, GG)                                                      \
+    if (cfg.K == KK && cfg.G == GG)                                                     \
+        return cfg.x_dtype == DENDSN_BF16 ? launch_forward_tp<KK, GG, 1>(a, cfg.psi, layout, s) \
+                                          : launch_forward_tp<KK, GG, 0>(a, cfg.psi, layout, s);
+#define DENDSN_TP_BWD_CASE(KK, GG)                                                      \
+    if (cfg.K == KK && cfg.G == GG)                                                     \
+        return cfg.x_dtype == DENDSN_BF16 ? launch_backward_tp<KK, GG, 1>(a, cfg.psi, layout, s) \
+                                          : launch_backward_tp<KK, GG, 0>(a, cfg.psi, layout, s);
+
+cudaError_t dispatch_forward_tp(const dendsn_config &cfg, int layout, const FwdArgs &a, cudaStream_t s) {
+    DENDSN_KG_LIST(DENDSN_TP_FWD_CASE)
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t dispatch_backward_tp(const dendsn_config &cfg, int layout, const BwdArgs &a, cudaStream_t s) {
+    DENDSN_KG_LIST(DENDSN_TP_BWD_CASE)
+    return cudaErrorInvalidValue;
+}
+
 }  // namespace
 
 extern "C" {
@@ -288,7 +316,8 @@ dendsn_status dendsn_forward(const dendsn_config *cfg, const void *x, const floa
     a.ck_vd = (saved && pl.gf.n_ck > 0) ? static_cast<float *>(saved) : nullptr;
     a.ck_vs = a.ck_vd ? reinterpret_cast<float *>(static_cast<char *>(saved) + pl.ck_vd_bytes)
                       : nullptr;
-    cudaError_t e = dispatch_forward(*cfg, pl.layout, a, pl.blocks_f, static_cast<cudaStream_t>(stream));
+    cudaError_t e = pl.tp ? dispatch_forward_tp(*cfg, pl.layout, a, static_cast<cudaStream_t>(stream))
+                          : dispatch_forward(*cfg, pl.layout, a, pl.blocks_f, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess)
         return fail(DENDSN_ERR_CUDA, "forward launch failed: %s", cudaGetErrorString(e));
     g_launches.fetch_add(1, std::memory_order_relaxed);
@@ -343,7 +372,8 @@ dendsn_status backward_impl(const dendsn_config *cfg, const void *x, const float
         a.gx = grad_x;
         a.partials = static_cast<float *>(scratch);
         a.want_beta = grad_beta != nullptr;
-        cudaError_t e = dispatch_backward(*cfg, pl.layout, pl.gb.L, a, pl.blocks_b, s);
+        cudaError_t e = pl.tp ? dispatch_backward_tp(*cfg, pl.layout, a, s)
+                              : dispatch_backward(*cfg, pl.layout, pl.gb.L, a, pl.blocks_b, s);
         if (e != cudaSuccess)
             return fail(DENDSN_ERR_CUDA, "backward launch failed: %s", cudaGetErrorString(e));
         g_launches.fetch_add(1, std::memory_order_relaxed);
@@ -357,7 +387,7 @@ dendsn_status backward_impl(const dendsn_config *cfg, const void *x, const float
     f.g_kappa = grad_kappa;
     f.g_beta = grad_beta;
     f.stateless = cfg->stateless;
-    cudaError_t e = launch_finalize(f, s);
+    cudaError_t e = pl.tp ? launch_finalize_tp(f, s) : launch_finalize(f, s);
     if (e != cudaSuccess)
         return fail(DENDSN_ERR_CUDA, "finalize launch failed: %s", cudaGetErrorString(e));
     g_launches.fetch_add(1, std::memory_order_relaxed);

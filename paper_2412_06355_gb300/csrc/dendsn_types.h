@@ -89,6 +89,19 @@ template <int K, int G, int PSI, int XT, int L, int LAYOUT>
 cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s);
 cudaError_t launch_finalize(const FinArgs &a, cudaStream_t s);
 
+// Time-parallel kernels (tp_kernels.cu): one warp per neuron, for layers with at least
+// kTpMinT steps and at most kTpMaxNeurons neurons whose backward history fits in shared
+// memory. XT: 0 = float, 1 = bfloat16; psi and layout are runtime arguments.
+constexpr int kTpMinT = 256;
+constexpr int64_t kTpMaxNeurons = 2048;
+constexpr size_t kTpMaxSmem = 200 * 1024;
+size_t tp_smem_bytes(int T, int K, bool backward);
+template <int K, int G, int XT>
+cudaError_t launch_forward_tp(const FwdArgs &a, int psi, int layout, cudaStream_t s);
+template <int K, int G, int XT>
+cudaError_t launch_backward_tp(const BwdArgs &a, int psi, int layout, cudaStream_t s);
+cudaError_t launch_finalize_tp(const FinArgs &a, cudaStream_t s);
+
 // Point-neuron LIF layer: x, spikes, gs, gx are [T, M] in the x dtype; v_out and gv
 // [T, M] float32; ck [(T + 7) / 8 - 1, M] float32 somatic potentials at the ends of
 // the 8-step chunks (T > 4 only).

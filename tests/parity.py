@@ -1,7 +1,7 @@
 """Shared machinery of the GPU-vs-oracle parity tests.
 
 Tolerances (written here once, used by every parity test):
-  V^s      |gpu - oracle| <= 1e-6 + 1e-5 |oracle|             (float32 state)
+  V^s      |gpu - oracle| <= 1e-6 + 1e-5 |oracle| (+ the soma allowance below)
   spikes   identical, except at and after a step where the oracle's potential lies
            within 1e-5 of the threshold (an "ambiguous" step: float32 rounding may
            legitimately decide it either way)
@@ -16,6 +16,16 @@ Tolerances (written here once, used by every parity test):
   themselves the soma's reverse scan (memory 1 / (1 - beta)), so its atol_rel is
   max(1e-5, eps32 / ((1 - alpha_max)(1 - beta))): 1e-5 for beta = 0.5, 2.4e-5 for the
   long-horizon layers with alpha, beta = 0.95 (~400 effective terms).
+
+V^s gets a per-element allowance on top of 1e-6 + 1e-5 |v|. The soma recursion
+V[t] = beta leak[t-1] + Z[t] (Eq. methods-lif-reset-charge) adds a float32 rounding of about
+eps32 (|Z[t]| + |V[t]|) per step and carries earlier ones with weight beta (cut by a hard
+reset), and Z[t] inherits the compartment scan's rounding (about eps32 sum_k alpha^k |X|)
+through kappa m |psi'| / zeta. With beta = 0.95 and a soft reset that reaches several 1e-6 where
+V^s itself is near zero, and a plain sequential float32 restatement misses the bare bound
+there too. The allowance is 2x that first-order error: a median 5e-7 on the beta = 0.5 conv
+layer (a tenth of the bare bound there). A step is ambiguous when the oracle's V^s lies within max(1e-5, that V^s tolerance)
+of theta.
 
 Neurons whose oracle trajectory has an ambiguous step get zero upstream gradient
 (grad_spikes and grad_v) on BOTH sides: the backward is linear in them, so those
@@ -71,15 +81,50 @@ def assert_close(name, got, want, rtol, atol_rel, mask=None, atol_abs=0.0):
             f"bound={bound.flat[i]:.3e} (rtol={rtol}, atol={atol:.3e})")
 
 
-def first_ambiguous_step(v_oracle: np.ndarray, theta: float) -> np.ndarray:
-    """Per neuron ([T, ...] input): index of the first ambiguous step, or T."""
-    amb = np.abs(v_oracle - theta) < AMBIGUOUS
+def first_ambiguous_step(v_oracle: np.ndarray, theta: float, v_tol=None) -> np.ndarray:
+    """Per neuron ([T, ...] input): index of the first ambiguous step, or T. v_tol: the V^s
+    tolerance per element (widens the window where it exceeds 1e-5)."""
+    window = AMBIGUOUS if v_tol is None else np.maximum(AMBIGUOUS, v_tol)
+    amb = np.abs(v_oracle - theta) < window
     T = v_oracle.shape[0]
     first = np.where(amb.any(axis=0), amb.argmax(axis=0), T)
     return first
 
 
 EPS32 = 2.0 ** -24
+
+
+def soma_rounding_allowance(w, x, chan, mrow, alpha, xi, zeta, kappa, mask, v_o):
+    """Extra V^s tolerance [T, M] (see above). x [T, M, K] float64, v_o the oracle's V^s [T, M]."""
+    T, M, K = x.shape
+    if T == 0 or M == 0:
+        return np.zeros((T, M))
+    G = w.G
+    f64 = lambda a: np.asarray(a.cpu() if hasattr(a, "cpu") else a, np.float64)
+    a = np.zeros((M, K)) if w.stateless else f64(alpha)[chan]
+    km = f64(kappa)[chan]
+    if mask is not None:
+        km = km * f64(mask)[mrow]
+    dpsi = 1.0 if w.psi == "identity" else 1.5          # max |psi'| (Mexican hat: ~1.38)
+    gain = np.repeat(np.abs(km) * dpsi / f64(zeta)[chan], G, axis=1)   # [M, K]
+    acc = np.zeros((M, K))
+    m = np.zeros(M)
+    v_prev = np.zeros(M)
+    s_prev = np.zeros(M, bool)
+    out = np.zeros((T, M))
+    for t in range(T):
+        acc = np.abs(x[t]) + a * acc
+        if w.reset == "soft":
+            leak, keep = v_prev - w.theta * s_prev, np.full(M, w.beta)
+        else:
+            leak, keep = np.where(s_prev, 0.0, v_prev), np.where(s_prev, 0.0, w.beta)
+        z = v_o[t] - w.beta * leak                          # Z[t], exactly, from the trajectory
+        m = keep * m + np.abs(z) + np.abs(v_o[t]) + (gain * acc).sum(axis=1)
+        if w.residual:
+            m = m + np.abs(x[t]).sum(axis=1) / K
+        out[t] = 2.0 * EPS32 * m
+        v_prev, s_prev = v_o[t], v_o[t] >= w.theta
+    return out
 
 
 def gx_atol_rel(w, alpha, base=G_ATOL_REL):
@@ -161,7 +206,13 @@ def check_layer(w, seed_inputs=None, with_gv=True):
     """Full parity check of workload `w` (all neurons) against the oracle."""
     inp = seed_inputs if seed_inputs is not None else workloads.make_inputs(w, "cpu", with_gv=with_gv)
     s_o, v_o = oracle.forward_layer(w, inp)
-    first = first_ambiguous_step(v_o, w.theta)              # [B, N]
+    chan, mrow = oracle.layer_channels(w.B, w.N, w.C, w.inner, w.mask_per_neuron)
+    xk = oracle.layer_x(w, inp["x"])
+    v_extra = soma_rounding_allowance(w, xk, chan, mrow, inp["alpha"], inp["xi"], inp["zeta"],
+                                      inp["kappa"], inp.get("mask"),
+                                      v_o.reshape(w.T, -1)).reshape(v_o.shape)
+    v_tol = V_ATOL + V_RTOL * np.abs(v_o) + v_extra
+    first = first_ambiguous_step(v_o, w.theta, v_tol)       # [B, N]
     amb = first < w.T
     gs = inp["gs"].clone()
     gs[:, torch.from_numpy(amb)] = 0
@@ -172,9 +223,8 @@ def check_layer(w, seed_inputs=None, with_gv=True):
     dev = to_dev(inp)
     got = run_gpu(w, dev, gs.cuda(), None if gv is None else gv.cuda())
     ref = oracle.backward_layer(w, dict(inp, gv=gv), gs=gs, want_dvs=True)
-    chan, mrow = oracle.layer_channels(w.B, w.N, w.C, w.inner, w.mask_per_neuron)
     extra = direction_rounding_allowance(
-        w, oracle.layer_x(w, inp["x"]), chan, mrow, inp["alpha"], inp["xi"], inp["zeta"],
+        w, xk, chan, mrow, inp["alpha"], inp["xi"], inp["zeta"],
         inp["kappa"], inp.get("mask"), ref["dvs"].reshape(w.T, w.B * w.N))
     if not np.isscalar(extra):
         extra = oracle.layer_gx(w, extra)
@@ -182,7 +232,7 @@ def check_layer(w, seed_inputs=None, with_gv=True):
     t_idx = np.arange(w.T)[:, None, None]
     v_mask = t_idx <= first[None]                           # V compared up to the first ambiguous step
     s_mask = t_idx < first[None]                            # S compared before it
-    assert_close("V^s", got["v"], v_o, V_RTOL, 0.0, mask=v_mask, atol_abs=V_ATOL)
+    assert_close("V^s", got["v"], v_o, V_RTOL, 0.0, mask=v_mask, atol_abs=V_ATOL + v_extra)
     assert np.array_equal(got["s"][s_mask], s_o[s_mask]), \
         f"spikes differ at {int((got['s'][s_mask] != s_o[s_mask]).sum())} unambiguous steps"
     assert set(np.unique(got["s"]).tolist()) <= {0.0, 1.0}

@@ -109,3 +109,35 @@ def test_random_lif(c):
     assert np.array_equal(oracle.to_f64(s)[sm], s_o[sm])
     rt, ar = (BF16_RTOL, BF16_ATOL_REL) if c["dtype"] == "bf16" else (G_RTOL, G_ATOL_REL)
     assert_close("grad_x", oracle.to_f64(gx), oracle.lif_backward(oc, inp["x"], gs, gv), rt, ar)
+
+
+# Layers that take the time-parallel kernels (at least 256 steps, at most 2048 neurons): the
+# compartment scans run in parallel over time there, so every flag is exercised again.
+def draw_tp_layer(i: int) -> workloads.Workload:
+    r = random.Random(9000 + i)
+    K, G = r.choice(KG)
+    inner = r.choice([1, 7, 32, 64])
+    C = r.choice([1, 2, 3])
+    per_sample = C * inner
+    N = per_sample * r.choice([1, 2])
+    B = r.choice([1, 2, 4])
+    T = r.choice([256, 257, 300, 640, 1000])
+    mask_p = r.choice([None, 0.5])
+    return workloads.Workload(
+        f"tp{i}", T=T, B=B, N=N, K=K, G=G, C=C, inner=inner,
+        dtype=r.choice(["f32", "f32", "bf16"]), psi=r.choice(["mh", "identity"]),
+        reset=r.choice(["hard", "soft"]), theta=r.choice([1.0, 0.6]),
+        beta=r.choice([0.5, 0.9, 0.95]), x_mean=r.choice([0.1, 0.3]),
+        x_density=r.choice([1.0, 0.3]), mask_p=mask_p,
+        mask_per_neuron=bool(mask_p is not None and r.random() < 0.5),
+        stateless=r.random() < 0.25, residual=r.random() < 0.25,
+        detach_reset=r.random() < 0.2, layout=r.choice(["kinner", "paper"]), seed=i)
+
+
+TP_LAYERS = [draw_tp_layer(i) for i in range(40)]
+
+
+@pytest.mark.parametrize("w", TP_LAYERS, ids=[_id(w) for w in TP_LAYERS])
+def test_random_time_parallel_layer(w):
+    assert binding.dendsn_workspace_size(binding.config_of(w))[0] == 0   # no checkpoints
+    check_layer(w)
