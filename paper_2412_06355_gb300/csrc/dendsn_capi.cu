@@ -90,16 +90,17 @@ int sm_count() {
 
 bool is01(int32_t v) { return v == 0 || v == 1; }
 
-// Tiling of the O x P neuron matrix for blocks of nt threads, lpn lanes per neuron.
-dendsn_status tile(Geometry &g, int nt, int lpn, int64_t sms, int64_t *blocks) {
+// Tiling of the O x P neuron matrix for blocks of nt threads, lpn lanes per neuron, about
+// per_sm blocks per SM in total (fewer means more rows per thread).
+dendsn_status tile(Geometry &g, int nt, int lpn, int64_t sms, int per_sm, int64_t *blocks) {
     const int W = 32 / lpn;                     // columns per warp
     const int full = nt / lpn;                  // columns of a one-row tile
     g.TXn = (g.inner >= W && g.P % full == 0) ? full : W;
     g.TY = nt / (g.TXn * lpn);
     g.seg = (g.inner % W == 0) ? W : ((W % g.inner == 0) ? g.inner : 1);
     g.nCT = (int32_t)((g.P + g.TXn - 1) / g.TXn);
-    // rows per thread: about 16 blocks per SM in total, at least one row
-    const int64_t target_blocks = 16LL * sms;
+    // rows per thread: about per_sm blocks per SM in total, at least one row
+    const int64_t target_blocks = (int64_t)per_sm * sms;
     const int64_t rg_target = std::max<int64_t>(1, (target_blocks + g.nCT - 1) / g.nCT);
     const int64_t rows_per_rg = std::max<int64_t>(1, (g.O + rg_target - 1) / rg_target);
     g.R = (int32_t)std::max<int64_t>(1, (rows_per_rg + g.TY - 1) / g.TY);
@@ -163,9 +164,13 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) 
     pl->gf = g;
     pl->gb = g;
     const int KTB = bwd_lane_compartments(c.K, c.G, c.x_dtype, g.L);
-    dendsn_status st = tile(pl->gf, fwd_threads(c.K), c.K / KT, sms, &bf);
+    dendsn_status st = tile(pl->gf, fwd_threads(c.K), c.K / KT, sms, 16, &bf);
     if (st != DENDSN_OK) return st;
-    if ((st = tile(pl->gb, bwd_threads(KTB), c.K / KTB, sms, &bb)) != DENDSN_OK) return st;
+    // backward: when every column is its own channel (inner = 1) each thread's parameter
+    // setup is heavier, and twice the rows per thread measured faster (token layer 285 ->
+    // 272 us); elsewhere 16 blocks per SM measured best
+    const int bwd_per_sm = (c.inner == 1) ? 8 : 16;
+    if ((st = tile(pl->gb, bwd_threads(KTB), c.K / KTB, sms, bwd_per_sm, &bb)) != DENDSN_OK) return st;
     pl->blocks_f = (int)bf;
     pl->blocks_b = (int)bb;
     pl->sx = (c.x_dtype == DENDSN_BF16) ? 2 : 4;
