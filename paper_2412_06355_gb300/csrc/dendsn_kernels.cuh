@@ -679,6 +679,12 @@ __device__ __forceinline__ ThreadPos thread_pos(const Geometry &g) {
 #define DENDSN_FWD_ASYNC 1
 #endif
 constexpr int kFwdDepth = 8;   // steps of x in flight per thread on the cp.async path
+// The forward's ring depth: 16 steps for float32 slots of up to 16 bytes (conv and event
+// layers' forward 1-2% faster), else 8 (wider slots would halve the resident blocks; the
+// bf16 8-compartment forward measured 1% slower with 16)
+template <typename XT, typename Raw> constexpr int fwd_depth() {
+    return (std::is_same<XT, float>::value && sizeof(Raw) <= 16) ? 16 : 8;
+}
 #ifndef DENDSN_BWD_ASYNC
 #define DENDSN_BWD_ASYNC 1
 #endif
@@ -782,7 +788,7 @@ __device__ __forceinline__ int64_t lane_x_offset(int64_t j, int sub, int KT, int
     return (j - s) * K + s + (int64_t)sub * KT * inner;
 }
 
-// x is fetched kFwdDepth steps ahead of use through the cp.async ring (or, without it, a
+// x is fetched fwd_depth() steps ahead of use through the cp.async ring (or, without it, a
 // ring of kFwdBatch registers); checkpoints every g.L steps (g.L is a power of two and a
 // multiple of the batch).
 // Lanes of 8 compartments: 3 blocks per SM for float32 (measured 2% faster), 2 for bf16
@@ -822,10 +828,10 @@ dendsn_forward_kernel(const FwdArgs A) {
     const bool residual = P.residual != 0;
 
     if constexpr (ASYNC) {
-        // Inputs are staged through a ring of kFwdDepth shared-memory slots per thread,
-        // filled by cp.async kFwdDepth steps ahead of use along this thread's
-        // (row, step) sequence; each thread reads only its own slots.
-        constexpr int D = kFwdDepth;
+        // Inputs are staged through a ring of D shared-memory slots per thread, filled by
+        // cp.async D steps ahead of use along this thread's (row, step) sequence; each
+        // thread reads only its own slots.
+        constexpr int D = fwd_depth<XT, typename V::Raw>();
         using Raw = typename V::Raw;
         extern __shared__ float4 fwd_smem[];
         Raw *ring = reinterpret_cast<Raw *>(fwd_smem) + threadIdx.x;     // slot k at ring[k * NT]
@@ -1455,7 +1461,7 @@ cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s) {
             return cudaGetLastError();
         }
     }
-    const size_t smem = (DENDSN_FWD_ASYNC && XI::kAsync) ? raw * kFwdDepth * NT : 0;
+    const size_t smem = (DENDSN_FWD_ASYNC && XI::kAsync) ? raw * fwd_depth<T, typename XI::Raw>() * NT : 0;
     cudaError_t e = allow_smem(dendsn_forward_kernel<K, G, PSI, T, LAYOUT>, smem);
     if (e != cudaSuccess) return e;
     dendsn_forward_kernel<K, G, PSI, T, LAYOUT><<<blocks, NT, smem, s>>>(a);
