@@ -115,7 +115,7 @@ dendsn_status tile(Geometry &g, int nt, int lpn, int64_t sms, int per_sm, int64_
     return DENDSN_OK;
 }
 
-dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) {
+dendsn_status make_plan(const dendsn_config *cfg, Plan *pl) {
     if (cfg == nullptr) return fail(DENDSN_ERR_INVALID_ARG, "cfg is NULL");
     const dendsn_config &c = *cfg;
     if (c.T < 0 || c.B < 0 || c.N < 0)
@@ -159,7 +159,7 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl, bool need_sm_count) 
     g.Kb = c.K / c.G;
     g.L = (c.T <= 4) ? 4 : 8;
     g.n_ck = (c.T > g.L) ? (c.T + g.L - 1) / g.L - 1 : 0;
-    const int64_t sms = need_sm_count ? sm_count() : 152;
+    const int64_t sms = sm_count();
     int64_t bf = 0, bb = 0;
     pl->gf = g;
     pl->gb = g;
@@ -291,7 +291,7 @@ extern "C" {
 dendsn_status dendsn_workspace_size(const dendsn_config *cfg, size_t *saved_bytes,
                                     size_t *scratch_bytes) {
     Plan pl;
-    dendsn_status st = make_plan(cfg, &pl, true);
+    dendsn_status st = make_plan(cfg, &pl);
     if (st != DENDSN_OK) return st;
     if (saved_bytes) *saved_bytes = pl.saved_bytes;
     if (scratch_bytes) *scratch_bytes = pl.scratch_bytes;
@@ -303,7 +303,7 @@ dendsn_status dendsn_forward(const dendsn_config *cfg, const void *x, const floa
                              const uint8_t *mask, void *spikes, float *v_out, void *saved,
                              void *stream) {
     Plan pl;
-    dendsn_status st = make_plan(cfg, &pl, true);
+    dendsn_status st = make_plan(cfg, &pl);
     if (st != DENDSN_OK) return st;
     if (pl.gf.BN == 0 || pl.gf.T == 0) return DENDSN_OK;
     if (!x || !spikes) return fail(DENDSN_ERR_INVALID_ARG, "x or spikes is NULL");
@@ -340,7 +340,7 @@ dendsn_status backward_impl(const dendsn_config *cfg, const void *x, const float
                             float *grad_alpha, float *grad_xi, float *grad_zeta,
                             float *grad_kappa, float *grad_beta, void *scratch, void *stream) {
     Plan pl;
-    dendsn_status st = make_plan(cfg, &pl, true);
+    dendsn_status st = make_plan(cfg, &pl);
     if (st != DENDSN_OK) return st;
     if (!grad_alpha || !grad_xi || !grad_zeta || !grad_kappa)
         return fail(DENDSN_ERR_INVALID_ARG, "parameter-gradient pointer is NULL");
@@ -492,7 +492,7 @@ extern "C" dendsn_status dendsn_backward_noalloc(
     const float *grad_v, const void *saved, void *grad_x, float *grad_alpha, float *grad_xi,
     float *grad_zeta, float *grad_kappa, void *stream) {
     Plan pl;
-    dendsn_status st = make_plan(cfg, &pl, true);
+    dendsn_status st = make_plan(cfg, &pl);
     if (st != DENDSN_OK) return st;
     if (pl.scratch_bytes > kNoAllocScratchBytes)
         return fail(DENDSN_ERR_UNSUPPORTED,
