@@ -370,3 +370,39 @@ def test_cuda_graph_capture_and_replay():
         assert torch.equal(gx, g["gx"])
         for got, k in zip(grads, ("galpha", "gxi", "gzeta", "gkappa")):
             assert torch.equal(got, g[k]), k
+
+
+def test_concurrent_streams_match_sequential_calls():
+    """Two layers (one of them on the time-parallel kernels) run at the same time on two streams
+    give the bits of running them one after the other: the library keeps no shared state."""
+    ws = [workloads.Workload("cs_a", T=9, B=4, N=4 * 256, K=4, G=1, C=4, inner=256, dtype="f32",
+                             psi="mh", reset="hard", mask_p=0.5, seed=61),
+          workloads.Workload("cs_b", T=300, B=2, N=8 * 32, K=8, G=2, C=8, inner=32,
+                             dtype="bf16", psi="identity", reset="soft", seed=62)]
+    cfgs = [binding.config_of(w) for w in ws]
+    inps = [to_dev(workloads.make_inputs(w, "cpu")) for w in ws]
+
+    def run(k, stream):
+        w, cfg, inp = ws[k], cfgs[k], inps[k]
+        saved, scratch = binding.workspace(cfg)
+        with torch.cuda.stream(stream):
+            s, _ = binding.forward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"],
+                                   inp["kappa"], inp["mask"], saved=saved, stream=stream)
+            g = binding.backward(cfg, inp["x"], inp["alpha"], inp["xi"], inp["zeta"],
+                                 inp["kappa"], inp["mask"], inp["gs"], None, saved, scratch,
+                                 stream=stream)
+        return s, g
+
+    ref = []
+    for k in range(2):
+        ref.append(run(k, torch.cuda.current_stream()))
+        torch.cuda.synchronize()
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    for st in streams:
+        st.wait_stream(torch.cuda.current_stream())
+    got = [run(k, streams[k]) for k in range(2)]
+    torch.cuda.synchronize()
+    for (s0, g0), (s1, g1) in zip(ref, got):
+        assert torch.equal(s0, s1)
+        for key in g0:
+            assert torch.equal(g0[key], g1[key]), key
