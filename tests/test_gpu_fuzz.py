@@ -141,3 +141,13 @@ TP_LAYERS = [draw_tp_layer(i) for i in range(40)]
 def test_random_time_parallel_layer(w):
     assert binding.dendsn_workspace_size(binding.config_of(w))[0] == 0   # no checkpoints
     check_layer(w)
+
+
+@pytest.mark.parametrize("reset", ["hard", "soft"])
+@pytest.mark.parametrize("theta", [0.0, -0.3])
+def test_time_parallel_nonpositive_threshold(reset, theta):
+    """theta <= 0: V^s[-1] = 0 already reaches the threshold, yet no spike precedes step 0."""
+    w = workloads.Workload("tp_theta", T=300, B=2, N=64, K=4, G=2, C=2, inner=32, dtype="f32",
+                           psi="mh", reset=reset, theta=theta, beta=0.8, seed=77)
+    assert binding.dendsn_workspace_size(binding.config_of(w))[0] == 0   # the time-parallel path
+    check_layer(w)
