@@ -267,14 +267,27 @@ __device__ __forceinline__ typename MaskRaw<KTb>::T fetch_neuron_mask(const Para
     return fetch_mask<KTb>(P.mask + n * g.Kb + sub * KTb);
 }
 
+// kappa * m and m of a lane's KTb branches from their raw mask bytes (nonzero: kept) and
+// kappa: a select, not a product (kappa * 1 = kappa, kappa * 0 = 0 up to the sign of zero).
 template <int KTb>
-__device__ __forceinline__ void apply_neuron_mask(const Params &P, const Geometry &g,
-                                                  const typename MaskRaw<KTb>::T &raw, int chan,
-                                                  int sub, float (&km)[KTb], float (&mk)[KTb]) {
-    unpack_mask<KTb>(raw, mk);
+__device__ __forceinline__ void apply_neuron_mask(const typename MaskRaw<KTb>::T &raw,
+                                                  const float (&kap)[KTb],
+                                                  float (&km)[KTb], float (&mk)[KTb]) {
 #pragma unroll
-    for (int b = 0; b < KTb; ++b)
-        km[b] = __fmul_rn(__ldg(P.kappa + (int64_t)chan * g.Kb + sub * KTb + b), mk[b]);
+    for (int b = 0; b < KTb; ++b) {
+        uint32_t w;
+        if constexpr (KTb == 8) w = b < 4 ? raw.x : raw.y;
+        else w = raw;
+        const bool on = (w & (0xffu << (8 * (b & 3)))) != 0u;
+        km[b] = on ? kap[b] : 0.f;
+        mk[b] = on ? 1.f : 0.f;
+    }
+}
+
+// Bytes of dynamic shared memory in front of a kernel's other regions that hold each
+// thread's KTb kappa values when masks are per neuron (else none).
+__host__ __device__ constexpr size_t kappa_smem_bytes(int mask_mode, int KTb, int NT) {
+    return mask_mode == 2 ? (size_t)KTb * NT * sizeof(float) : 0;
 }
 
 // ================================================================ paired engine, G = 1
@@ -303,9 +316,9 @@ struct PairArith {
     static __device__ __forceinline__ MRaw fetch_neuron_mask(const Params &P, const Geometry &g, int64_t n, int sub) {
         return dendsn::fetch_neuron_mask<KT>(P, g, n, sub);
     }
-    static __device__ __forceinline__ void neuron_mask(const Params &P, const Geometry &g, const MRaw &raw, int chan, int sub, LP &lp) {
+    static __device__ __forceinline__ void neuron_mask(const MRaw &raw, const float (&kap)[KT], LP &lp) {
         float km[KT], mk[KT];
-        apply_neuron_mask<KT>(P, g, raw, chan, sub, km, mk);
+        apply_neuron_mask<KT>(raw, kap, km, mk);
 #pragma unroll
         for (int m = 0; m < N2; ++m) {
             lp.km[m] = make_float2(km[2 * m], km[2 * m + 1]);
@@ -462,8 +475,8 @@ struct ScalarArith {
     static __device__ __forceinline__ MRaw fetch_neuron_mask(const Params &P, const Geometry &g, int64_t n, int sub) {
         return dendsn::fetch_neuron_mask<KTb>(P, g, n, sub);
     }
-    static __device__ __forceinline__ void neuron_mask(const Params &P, const Geometry &g, const MRaw &raw, int chan, int sub, LP &lp) {
-        apply_neuron_mask<KTb>(P, g, raw, chan, sub, lp.km, lp.mk);
+    static __device__ __forceinline__ void neuron_mask(const MRaw &raw, const float (&kap)[KTb], LP &lp) {
+        apply_neuron_mask<KTb>(raw, kap, lp.km, lp.mk);
     }
     static __device__ __forceinline__ void zero(St &s) {
 #pragma unroll
@@ -591,23 +604,49 @@ using Arith = typename std::conditional<(G == 1 && KT % 2 == 0),
                                         ScalarArith<KT, G, PSI>>::type;
 
 // Per-neuron branch masks (mask_mode 2) of a thread's rows, each fetched one row ahead of
-// its use so the row start does not wait on the load. n: the neuron (within a sample) of
-// the next row; step: the thread's row stride in neurons, modulo N.
-template <typename AR>
+// its use so the row start does not wait on the load. kappa * m is rebuilt at each row
+// from the lane's kappa, copied once into the front of the block's dynamic shared memory
+// (kappa_smem_bytes: vectors of W values, vector v of thread i at [v * NT + i]) rather than
+// re-read from global memory per row. n: the neuron (within a sample) of the next row;
+// step: the thread's row stride in neurons, modulo N.
+template <typename AR, int NT>
 struct MaskAhead {
+    static constexpr int KTb = AR::KTb;
+    static constexpr int W = KTb % 4 == 0 ? 4 : (KTb % 2 == 0 ? 2 : 1);
+    using KV = typename std::conditional<W == 4, float4,
+                                         typename std::conditional<W == 2, float2, float>::type>::type;
     typename AR::MRaw next;
+    KV *kap;
     int n, step;
     __device__ __forceinline__ void init(const Params &P, const Geometry &g, int64_t j0,
-                                         int64_t jstep, int sub, int nrows) {
+                                         int64_t jstep, int chan, int sub, int nrows,
+                                         void *kbase) {
         n = (int)(j0 % g.N);
         step = (int)(jstep % g.N);
-        if (P.mask_mode == 2 && nrows > 0) next = AR::fetch_neuron_mask(P, g, n, sub);
+        kap = reinterpret_cast<KV *>(kbase) + threadIdx.x;
+        if (P.mask_mode != 2) return;
+        const float *src = P.kappa + (int64_t)chan * g.Kb + sub * KTb;
+#pragma unroll
+        for (int v = 0; v < KTb / W; ++v) {
+            KV q;
+#pragma unroll
+            for (int w = 0; w < W; ++w) reinterpret_cast<float *>(&q)[w] = __ldg(src + v * W + w);
+            kap[v * NT] = q;
+        }
+        if (nrows > 0) next = AR::fetch_neuron_mask(P, g, n, sub);
     }
     // applies the current row's mask, then requests the next row's (if `more`)
-    __device__ __forceinline__ void advance(const Params &P, const Geometry &g, int chan, int sub,
+    __device__ __forceinline__ void advance(const Params &P, const Geometry &g, int sub,
                                             bool more, typename AR::LP &lp) {
         if (P.mask_mode != 2) return;
-        AR::neuron_mask(P, g, next, chan, sub, lp);
+        float k[KTb];
+#pragma unroll
+        for (int v = 0; v < KTb / W; ++v) {
+            const KV q = kap[v * NT];
+#pragma unroll
+            for (int w = 0; w < W; ++w) k[v * W + w] = reinterpret_cast<const float *>(&q)[w];
+        }
+        AR::neuron_mask(next, k, lp);
         n += step;
         if (n >= g.N) n -= g.N;
         if (more) next = AR::fetch_neuron_mask(P, g, n, sub);
@@ -791,11 +830,10 @@ __device__ __forceinline__ int64_t lane_x_offset(int64_t j, int sub, int KT, int
 // x is fetched fwd_depth() steps ahead of use through the cp.async ring (or, without it, a
 // ring of kFwdBatch registers); checkpoints every g.L steps (g.L is a power of two and a
 // multiple of the batch).
-// Lanes of 8 compartments: 3 blocks per SM for float32 (measured 2% faster), 2 for bf16
-// (whose unpacking spills under the tighter cap, 15% slower).
+// Lanes of 8 compartments: 2 blocks per SM (the 3-block register cap spills: bf16 15%
+// slower, float32 with per-neuron masks 4% slower, float32 without them 1% slower).
 template <int K, int G, int PSI, typename XT, int LAYOUT>
-__global__ void __launch_bounds__(fwd_threads(K), lane_compartments(K) >= 8 ? (xt_code<XT>() == 0 ? 3 : 2)
-                                                                           : DENDSN_FWD_MINB)
+__global__ void __launch_bounds__(fwd_threads(K), lane_compartments(K) >= 8 ? 2 : DENDSN_FWD_MINB)
 dendsn_forward_kernel(const FwdArgs A) {
     constexpr int NT = fwd_threads(K);
     constexpr int KT = lane_compartments(K);
@@ -833,8 +871,11 @@ dendsn_forward_kernel(const FwdArgs A) {
         // thread reads only its own slots.
         constexpr int D = fwd_depth<XT, typename V::Raw>();
         using Raw = typename V::Raw;
+        // dynamic shared memory: the lanes' kappa (per-neuron masks only), then the ring
         extern __shared__ float4 fwd_smem[];
-        Raw *ring = reinterpret_cast<Raw *>(fwd_smem) + threadIdx.x;     // slot k at ring[k * NT]
+        Raw *ring = reinterpret_cast<Raw *>(reinterpret_cast<char *>(fwd_smem) +
+                                            kappa_smem_bytes(P.mask_mode, AR::KTb, NT)) +
+                    threadIdx.x;                                          // slot k at ring[k * NT]
         const XT *ip = xrow;                    // next step to fetch
         int it = 0, ir = 0;                     // its step and row
         const int64_t row_jump = rX - (int64_t)T * sX;
@@ -858,10 +899,10 @@ dendsn_forward_kernel(const FwdArgs A) {
             const XT *xr = xrow;
             XT *sr = srow;
             float *vr = vrow;
-            MaskAhead<AR> mask;
-            mask.init(P, g, j0, jstep, pos.sub, pos.nrows);
+            MaskAhead<AR, NT> mask;
+            mask.init(P, g, j0, jstep, pos.chan, pos.sub, pos.nrows, fwd_smem);
             for (int i = 0; i < pos.nrows; ++i) {
-                mask.advance(P, g, pos.chan, pos.sub, i + 1 < pos.nrows, lp);
+                mask.advance(P, g, pos.sub, i + 1 < pos.nrows, lp);
                 typename AR::St vd;
                 AR::zero(vd);
                 float v = 0.f;
@@ -936,10 +977,11 @@ dendsn_forward_kernel(const FwdArgs A) {
         }
     }
     int64_t j = j0;
-    MaskAhead<AR> mask;
-    mask.init(P, g, j0, jstep, pos.sub, pos.nrows);
+    extern __shared__ float4 fwd_smem[];         // the lanes' kappa (per-neuron masks only)
+    MaskAhead<AR, NT> mask;
+    mask.init(P, g, j0, jstep, pos.chan, pos.sub, pos.nrows, fwd_smem);
     for (int i = 0; i < pos.nrows; ++i) {
-        mask.advance(P, g, pos.chan, pos.sub, i + 1 < pos.nrows, lp);
+        mask.advance(P, g, pos.sub, i + 1 < pos.nrows, lp);
         typename AR::St vd;
         AR::zero(vd);
         float v = 0.f;
@@ -1031,9 +1073,12 @@ dendsn_forward_staged_kernel(const FwdArgs A) {
     const bool write_ck = (A.ck_vd != nullptr) && g.n_ck > 0;
     const bool residual = P.residual != 0;
 
+    // dynamic shared memory: the lanes' kappa (per-neuron masks only), then the slots
     extern __shared__ float4 fwd_smem[];
     constexpr int kSlot = NT * K;                // elements of one slot (all warps)
-    XT *wring = reinterpret_cast<XT *>(fwd_smem) + (threadIdx.x >> 5) * (32 * K);
+    XT *wring = reinterpret_cast<XT *>(reinterpret_cast<char *>(fwd_smem) +
+                                       kappa_smem_bytes(P.mask_mode, AR::KTb, NT)) +
+                (threadIdx.x >> 5) * (32 * K);
     int64_t src[CPL];
     int dst[CPL];
 #pragma unroll
@@ -1064,10 +1109,10 @@ dendsn_forward_staged_kernel(const FwdArgs A) {
     }
     int slot = 0;
     int64_t j = j0;
-    MaskAhead<AR> mask;
-    mask.init(P, g, j0, jstep, 0, pos.nrows);
+    MaskAhead<AR, NT> mask;
+    mask.init(P, g, j0, jstep, pos.chan, 0, pos.nrows, fwd_smem);
     for (int i = 0; i < pos.nrows; ++i) {
-        mask.advance(P, g, pos.chan, 0, i + 1 < pos.nrows, lp);
+        mask.advance(P, g, 0, i + 1 < pos.nrows, lp);
         typename AR::St vd;
         AR::zero(vd);
         float v = 0.f;
@@ -1170,8 +1215,11 @@ dendsn_backward_kernel(const BwdArgs A) {
     const bool residual = P.residual != 0;
     const bool has_gv = A.gv != nullptr;
 
+    // dynamic shared memory: the lanes' kappa (per-neuron masks only), then the history,
+    // V^s history and x ring, or (at the end) the reduction
     extern __shared__ float4 smem_f4[];
-    HistRaw *hist = reinterpret_cast<HistRaw *>(smem_f4);                             // [L][NT]
+    char *const sregion = reinterpret_cast<char *>(smem_f4) + kappa_smem_bytes(P.mask_mode, KTb, NT);
+    HistRaw *hist = reinterpret_cast<HistRaw *>(sregion);                             // [L][NT]
     float *hist_vs = reinterpret_cast<float *>(hist + (SHIST ? L * NT : 0));   // [L][NT]
     XRaw *xring = reinterpret_cast<XRaw *>(hist_vs + (SHIST ? L * NT : 0)) + threadIdx.x;   // [D][NT]
     // cp.async walker over this thread's sequence: rows, chunks in reverse, steps forward
@@ -1230,10 +1278,10 @@ dendsn_backward_kernel(const BwdArgs A) {
     }
 
     int64_t j = j0;
-    MaskAhead<AR> mask;
-    mask.init(P, g, j0, jstep, pos.sub, pos.nrows);
+    MaskAhead<AR, NT> mask;
+    mask.init(P, g, j0, jstep, pos.chan, pos.sub, pos.nrows, smem_f4);
     for (int i = 0; i < pos.nrows; ++i) {
-        mask.advance(P, g, pos.chan, pos.sub, i + 1 < pos.nrows, lp);
+        mask.advance(P, g, pos.sub, i + 1 < pos.nrows, lp);
         typename AR::St Ad;           // dL/dV^d[t+1], carried backwards
         AR::zero(Ad);
         float dvn = 0.f;              // dL/dV^s[t+1]
@@ -1400,7 +1448,7 @@ dendsn_backward_kernel(const BwdArgs A) {
             v[a] = __fadd_rn(v[a], __shfl_xor_sync(0xffffffffu, v[a], d * LPN));
     }
     // stage 2: run leaders meet in shared memory; red[a][tid] (reuses the history space)
-    float *red = reinterpret_cast<float *>(smem_f4);
+    float *red = reinterpret_cast<float *>(sregion);
     if constexpr (BASYNC) cp_async_wait<0>();
     __syncthreads();
 #pragma unroll
@@ -1454,14 +1502,16 @@ cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s) {
     if constexpr (LAYOUT == 1 && K >= 2 && K <= 8 && DENDSN_FWD_ASYNC) {
         // the paper layout with warps of 32 consecutive positions: staged per warp
         if (a.g.inner % 32 == 0 && a.g.TXn % 32 == 0) {
-            const size_t smem = (size_t)kFwdDepth * NT * K * sizeof(T);
+            const size_t smem = (size_t)kFwdDepth * NT * K * sizeof(T) +
+                                kappa_smem_bytes(a.p.mask_mode, K / G, NT);
             cudaError_t e = allow_smem(dendsn_forward_staged_kernel<K, G, PSI, T>, smem);
             if (e != cudaSuccess) return e;
             dendsn_forward_staged_kernel<K, G, PSI, T><<<blocks, NT, smem, s>>>(a);
             return cudaGetLastError();
         }
     }
-    const size_t smem = (DENDSN_FWD_ASYNC && XI::kAsync) ? raw * fwd_depth<T, typename XI::Raw>() * NT : 0;
+    const size_t smem = ((DENDSN_FWD_ASYNC && XI::kAsync) ? raw * fwd_depth<T, typename XI::Raw>() * NT : 0) +
+                        kappa_smem_bytes(a.p.mask_mode, KT / G, NT);
     cudaError_t e = allow_smem(dendsn_forward_kernel<K, G, PSI, T, LAYOUT>, smem);
     if (e != cudaSuccess) return e;
     dendsn_forward_kernel<K, G, PSI, T, LAYOUT><<<blocks, NT, smem, s>>>(a);
@@ -1479,7 +1529,8 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
     using XI = XIO<T, KT, LAYOUT>;
     constexpr size_t xraw = sizeof(typename XI::Raw);
     const size_t ring = (DENDSN_BWD_ASYNC && shist && XI::kAsync) ? xraw * kBwdDepth * NT : 0;
-    const size_t smem = red > hist + ring ? red : hist + ring;
+    const size_t smem = (red > hist + ring ? red : hist + ring) +
+                        kappa_smem_bytes(a.p.mask_mode, KT / G, NT);
     if (a.want_beta) {
         cudaError_t e = allow_smem(dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, true>, smem);
         if (e != cudaSuccess) return e;

@@ -45,8 +45,12 @@ struct TpParams {
     float a[K], nxi[K], iz[Kb], km[Kb], mk[Kb];
     __device__ __forceinline__ void load(const Params &P, const Geometry &g, int64_t n, int chan) {
         load_param_arrays<K, G>(P, g, chan, 0, a, nxi, iz, km, mk);
-        if (P.mask_mode == 2)
-            apply_neuron_mask<Kb>(P, g, fetch_neuron_mask<Kb>(P, g, n, 0), chan, 0, km, mk);
+        if (P.mask_mode == 2) {
+            float kap[Kb];                       // km holds kappa itself here (mk = 1)
+#pragma unroll
+            for (int b = 0; b < Kb; ++b) kap[b] = km[b];
+            apply_neuron_mask<Kb>(fetch_neuron_mask<Kb>(P, g, n, 0), kap, km, mk);
+        }
     }
 };
 
