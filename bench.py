@@ -31,6 +31,8 @@ UNIT = "neuron-steps/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 L2_BYTES = 129 * 2**20
+FP32_LANES_PER_SM = 128          # float32 FMA lanes per Blackwell SM
+NOMINAL_SM_MHZ = 2070.0
 
 
 def log(*a):
@@ -545,13 +547,25 @@ def run_ours(args):
 
     # ---- roofline of the dominant kernel
     ab = w.algorithmic_bytes()
+    ops = w.fp32_ops_per_neuron_step()
     fwd_avg, bwd_avg = statistics.mean(fwd_ms), statistics.mean(bwd_ms)
     peak, peak_kind = measured_hbm_peak()
     if bwd_avg >= fwd_avg:
-        kname, kbytes, kms = "dendsn_backward_kernel", ab["backward"], bwd_avg
+        kname, kbytes, kms, kops = "dendsn_backward_kernel", ab["backward"], bwd_avg, ops["backward"]
     else:
-        kname, kbytes, kms = "dendsn_forward_kernel", ab["forward"], fwd_avg
+        kname, kbytes, kms, kops = "dendsn_forward_kernel", ab["forward"], fwd_avg, ops["forward"]
     achieved = kbytes / (kms / 1e3) / 1e9
+    # the float32 roof of the same kernel: its float32 operations (a cost model counted from
+    # the equations) against SMs x 128 FMA lanes x the SM clock
+    sm_mhz = (clock or {}).get("sm_max_mhz") or NOMINAL_SM_MHZ
+    fp32_peak = torch.cuda.get_device_properties(dev).multi_processor_count * FP32_LANES_PER_SM * sm_mhz * 1e6
+    ops_launch = kops * w.neuron_steps
+    t_hbm, t_alu = kbytes / (peak * 1e9), ops_launch / fp32_peak
+    alu = {"fp32_ops_per_neuron_step": kops, "fp32_ops_per_launch": ops_launch,
+           "achieved_tops": ops_launch / (kms / 1e3) / 1e12, "peak_tops": fp32_peak / 1e12,
+           "frac": ops_launch / (kms / 1e3) / fp32_peak,
+           "peak_basis": f"SMs x {FP32_LANES_PER_SM} FP32 lanes x {sm_mhz:.0f} MHz",
+           "min_ms_at_fp32_peak": t_alu * 1e3, "min_ms_at_hbm_peak": t_hbm * 1e3}
     step_ms = ms / args.steps
     value = world * w.neuron_steps / (step_ms / 1e3)
     cpu = None
@@ -585,8 +599,14 @@ def run_ours(args):
             "parallelism": f"dp{world}" if world > 1 else "single GPU",
             "soma": "plif (learnable beta)" if args.plif else "lif",
             "launch": "cuda graph replay" if args.graph else "eager"}),
-        "roofline": {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peak,
-                     "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+        "roofline": {**({"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peak,
+                         "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak}
+                        if t_hbm >= t_alu else
+                        {"bound": "alu", "kernel": kname, "achieved": alu["achieved_tops"],
+                         "peak": alu["peak_tops"], "peak_kind": alu["peak_basis"],
+                         "unit": "FP32 Top/s", "frac": alu["frac"]}),
+                     "hbm_frac": achieved / peak,
+                     "alu": alu,
                      # counters were taken on the plain backward build, not the dL/dbeta one
                      "traffic": None if args.plif else recorded_traffic(kname, w.name),
                      "algorithmic_bytes_per_launch": kbytes, "avg_launch_ms": kms},

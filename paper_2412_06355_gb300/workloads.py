@@ -85,6 +85,43 @@ class Workload:
         bwd = ns * (self.K * s + s + self.K * s)
         return {"forward": fwd, "backward": bwd, "total": fwd + bwd}
 
+    def fp32_ops_per_neuron_step(self) -> dict:
+        """Float32 arithmetic a fused forward+backward needs per neuron-step, by kernel: a
+        cost model counted from the equations (a fused multiply-add is one operation; 1/zeta
+        and -xi/zeta are folded into the parameters once; exp2, sqrt and 1/x run on the
+        special-function unit and are counted apart, in `sfu`). Address arithmetic, loads,
+        stores, conversions, selects and compares other than the threshold are the
+        implementation's, not counted.
+
+        forward: per compartment V^d (Eq. methods-compartment; none when Stateless),
+        u = V^d/zeta - xi/zeta and its square (Eq. methods-branch-aggregation; for G = 1 the
+        identity branch needs only |u|, for G > 1 it takes a square root), the residual
+        term; per branch psi (Mexican hat: the exponent's scale and (1 - r^2) e, Eq.
+        methods-mexican-hat) and the kappa*m sum (Eq. methods-soma-input); per neuron the
+        charge and the threshold (+1 for the soft reset).
+        backward: the forward's recompute, then the reverse step: u and r^2 again; the soma
+        adjoint (dV[t+1]/dS, dL/dS, the surrogate's argument, square and + 1, dL/dV^s: 7,
+        Eq. methods-sg); per branch dL/dY, psi' (Mexican hat: the exponent's scale, y,
+        r^2 - 3, two products: 5; psi'(r)/r needs no 1/r), dr/du (G = 1: one product per
+        branch; G > 1: one per compartment, plus 1/r and a product per branch for the
+        identity), dzeta (2) and dkappa (2); per compartment dL/dV^d, dxi, the residual
+        gradient, and (Stateful) the reverse scan and dalpha.
+        """
+        K, Kb, G = self.K, self.Kb, self.G
+        mh = self.psi == "mh"
+        stateful = not self.stateless
+        square = K if (mh or G > 1) else 0
+        fwd = ((K if stateful else 0) + K + square + (K if self.residual else 0)
+               + Kb * ((2 if mh else 0) + 1)
+               + 2 + (1 if self.reset == "soft" else 0))
+        drdu = Kb if G == 1 else K + (0 if mh else Kb)
+        rev = (K + square + 7 + Kb * (1 + (5 if mh else 0) + 2 + 2) + drdu
+               + K * (1 + 1 + (2 if stateful else 0)) + (K if self.residual else 0))
+        sfu_f = Kb if (mh or G > 1) else 0
+        sfu_b = sfu_f + 1 + (Kb if (mh or G > 1) else 0)
+        return {"forward": fwd, "backward": fwd + rev,
+                "sfu": {"forward": sfu_f, "backward": sfu_b}}
+
     def with_(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)
 
