@@ -292,13 +292,25 @@ __host__ __device__ constexpr size_t kappa_smem_bytes(int mask_mode, int KTb, in
 
 // ================================================================ paired engine, G = 1
 // Compartment i is branch i. u = V^d/zeta - xi/zeta; r = |u|.
+// In the backward the branch mask enters the Mexican hat through its exponent: lm = 0 for
+// a kept branch and -inf for a masked one, so e^{-r^2/2} (and with it Y and psi') is
+// exactly 0 where m = 0 at no extra instruction; for the identity lm holds m itself. (The
+// forward needs no masked Y: kappa m = 0 already removes the branch from Z.)
+// The backward carries the dendritic adjoint and three of its sums without the factor
+// 1/zeta of Eq. methods-branch-aggregation (a per-lane constant): Ad' = zeta Ad, and
+// dL/dalpha, dL/dxi, dL/dzeta are scaled by 1/zeta once, in acc_export.
 template <int KT, int PSI, bool TREE>
 struct PairArith {
     static constexpr int N2 = KT / 2;
     static constexpr int KTb = KT;
-    struct LP { float2 a[N2], nxi[N2], iz[N2], km[N2], mk[N2]; };
+    struct LP { float2 a[N2], nxi[N2], iz[N2], km[N2], lm[N2]; };
     struct St { float2 v[N2]; };
     struct Acc { float2 ga[N2], ngxi[N2], ngz[N2], gk[N2]; };   // ngxi, ngz: negated sums
+    // mask value as the engine keeps it (see above)
+    static __device__ __forceinline__ float mask_term(float m) {
+        if constexpr (PSI == PSI_MEXHAT) return m != 0.f ? 0.f : -INFINITY;
+        else return m;
+    }
 
     static __device__ __forceinline__ void load(const Params &P, const Geometry &g, int chan, int sub, LP &lp) {
         float a[KT], nxi[KT], iz[KT], km[KT], mk[KT];
@@ -309,7 +321,7 @@ struct PairArith {
             lp.nxi[m] = make_float2(nxi[2 * m], nxi[2 * m + 1]);
             lp.iz[m] = make_float2(iz[2 * m], iz[2 * m + 1]);
             lp.km[m] = make_float2(km[2 * m], km[2 * m + 1]);
-            lp.mk[m] = make_float2(mk[2 * m], mk[2 * m + 1]);
+            lp.lm[m] = make_float2(mask_term(mk[2 * m]), mask_term(mk[2 * m + 1]));
         }
     }
     using MRaw = typename MaskRaw<KTb>::T;
@@ -322,7 +334,7 @@ struct PairArith {
 #pragma unroll
         for (int m = 0; m < N2; ++m) {
             lp.km[m] = make_float2(km[2 * m], km[2 * m + 1]);
-            lp.mk[m] = make_float2(mk[2 * m], mk[2 * m + 1]);
+            lp.lm[m] = make_float2(mask_term(mk[2 * m]), mask_term(mk[2 * m + 1]));
         }
     }
     static __device__ __forceinline__ void zero(St &s) {
@@ -411,51 +423,54 @@ struct PairArith {
 #pragma unroll
         for (int m = 0; m < N2; ++m) { c.ga[m] = f2(0.f); c.ngxi[m] = f2(0.f); c.ngz[m] = f2(0.f); c.gk[m] = f2(0.f); }
     }
-    // [alpha KT | xi KT | zeta KTb | kappa KTb]
-    static __device__ __forceinline__ void acc_export(const Acc &c, float *v) {
+    // [alpha KT | xi KT | zeta KTb | kappa KTb]; the first three carry the factor 1/zeta here
+    static __device__ __forceinline__ void acc_export(const LP &lp, const Acc &c, float *v) {
 #pragma unroll
         for (int m = 0; m < N2; ++m) {
-            v[2 * m] = c.ga[m].x;                v[2 * m + 1] = c.ga[m].y;
-            v[KT + 2 * m] = -c.ngxi[m].x;        v[KT + 2 * m + 1] = -c.ngxi[m].y;
-            v[2 * KT + 2 * m] = -c.ngz[m].x;     v[2 * KT + 2 * m + 1] = -c.ngz[m].y;
+            const float2 ga = fmul2(c.ga[m], lp.iz[m]);
+            const float2 gxi = fmul2(c.ngxi[m], lp.iz[m]);
+            const float2 gz = fmul2(c.ngz[m], lp.iz[m]);
+            v[2 * m] = ga.x;                     v[2 * m + 1] = ga.y;
+            v[KT + 2 * m] = -gxi.x;              v[KT + 2 * m + 1] = -gxi.y;
+            v[2 * KT + 2 * m] = -gz.x;           v[2 * KT + 2 * m + 1] = -gz.y;
             v[3 * KT + 2 * m] = c.gk[m].x;       v[3 * KT + 2 * m + 1] = c.gk[m].y;
         }
     }
-    // One reverse step: V^d[t] (vdt), V^d[t-1] (vdp) and dL/dZ[t] (dz) update the
-    // dendritic adjoint Ad = dL/dV^d (reverse scan of Eq. methods-compartment), the
-    // parameter-gradient partials, and give dL/dX[t] = Ad (+ res).
+    // One reverse step: V^d[t] (vdt), V^d[t-1] (vdp) and dL/dZ[t] (dz) update the scaled
+    // dendritic adjoint Ad' = zeta dL/dV^d (reverse scan of Eq. methods-compartment), the
+    // parameter-gradient partials, and give dL/dX[t] = Ad' / zeta + res.
+    // Per branch (G = 1): dL/du = kappa m dz psi'(u) with psi'(u) = u (u^2 - 3) e^{-u^2/2}
+    // (the Mexican hat of |u| is smooth in u) or sign(u) (identity); the direct term of
+    // dL/dV^d is dL/du / zeta; du/dxi = -1/zeta; du/dzeta = -u / zeta.
     static __device__ __forceinline__ void backward(const LP &lp, const St &vdt, const St &vdp, float dz,
                                                     St &Ad, Acc &acc, float res, float (&gx)[KT]) {
         const float2 dz2 = f2(dz);
+        const float2 res2 = f2(res);
 #pragma unroll
         for (int m = 0; m < N2; ++m) {
             const float2 u = ffma2(vdt.v[m], lp.iz[m], lp.nxi[m]);
             const float2 gy = fmul2(lp.km[m], dz2);              // dL/dY
-            float2 y, d, grr;                                    // Y, dL/dV^d direct, (dL/dr) r
+            float2 y, du;                                        // m Y, dL/du
             if constexpr (PSI == PSI_MEXHAT) {
                 const float2 ss = fmul2(u, u);
-                const float2 t = fmul2(f2(kNegHalfLog2e), ss);
+                const float2 t = ffma2(f2(kNegHalfLog2e), ss, lp.lm[m]);
                 const float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
                 y = ffma2(neg2(ss), e, e);
-                // psi'(r) / r = (r^2 - 3) e^{-r^2/2}: du = q u
-                const float2 q = fmul2(fmul2(fadd2(ss, f2(-3.f)), e), gy);
-                d = fmul2(fmul2(q, u), lp.iz[m]);
-                grr = fmul2(ss, q);
+                const float2 w = fmul2(fadd2(ss, f2(-3.f)), e);  // psi'(r) / r
+                du = fmul2(fmul2(w, u), gy);
             } else {
-                const float2 r = make_float2(fabsf(u.x), fabsf(u.y));
-                const float2 gu = make_float2(u.x > 0.f ? gy.x : (u.x < 0.f ? -gy.x : 0.f),
-                                              u.y > 0.f ? gy.y : (u.y < 0.f ? -gy.y : 0.f));
-                y = r;
-                d = fmul2(gu, lp.iz[m]);
-                grr = fmul2(gy, r);
+                y = fmul2(lp.lm[m], make_float2(fabsf(u.x), fabsf(u.y)));
+                du = make_float2(u.x > 0.f ? gy.x : (u.x < 0.f ? -gy.x : 0.f),
+                                 u.y > 0.f ? gy.y : (u.y < 0.f ? -gy.y : 0.f));
             }
-            acc.ngxi[m] = fadd2(acc.ngxi[m], d);                 // dxi = -direct
-            acc.ngz[m] = ffma2(grr, lp.iz[m], acc.ngz[m]);       // dzeta = -(dL/dr) r / zeta
-            acc.gk[m] = ffma2(fmul2(lp.mk[m], y), dz2, acc.gk[m]);
-            Ad.v[m] = ffma2(lp.a[m], Ad.v[m], d);
-            acc.ga[m] = ffma2(Ad.v[m], vdp.v[m], acc.ga[m]);
-            gx[2 * m] = __fadd_rn(Ad.v[m].x, res);
-            gx[2 * m + 1] = __fadd_rn(Ad.v[m].y, res);
+            acc.ngxi[m] = fadd2(acc.ngxi[m], du);                // zeta dxi = -sum du
+            acc.ngz[m] = ffma2(u, du, acc.ngz[m]);               // zeta dzeta = -sum u du
+            acc.gk[m] = ffma2(y, dz2, acc.gk[m]);                // dkappa = sum m Y dz
+            Ad.v[m] = ffma2(lp.a[m], Ad.v[m], du);
+            acc.ga[m] = ffma2(Ad.v[m], vdp.v[m], acc.ga[m]);     // zeta dalpha
+            const float2 g = ffma2(Ad.v[m], lp.iz[m], res2);
+            gx[2 * m] = g.x;
+            gx[2 * m + 1] = g.y;
         }
     }
 };
@@ -531,7 +546,7 @@ struct ScalarArith {
 #pragma unroll
         for (int b = 0; b < KTb; ++b) { c.gz[b] = 0.f; c.gk[b] = 0.f; }
     }
-    static __device__ __forceinline__ void acc_export(const Acc &c, float *v) {
+    static __device__ __forceinline__ void acc_export(const LP &, const Acc &c, float *v) {
 #pragma unroll
         for (int i = 0; i < KT; ++i) { v[i] = c.ga[i]; v[KT + i] = c.gxi[i]; }
 #pragma unroll
@@ -1163,7 +1178,10 @@ constexpr int acc_count() { return 2 * KT + 2 * (KT / G); }
 
 // BETA: also accumulate dL/dbeta (a learnable somatic decay); a separate instance because
 // even one more live accumulator slows the register-history path measurably.
-template <int K, int G, int PSI, typename XT, int L, int LAYOUT, bool BETA>
+// FULL: T is a multiple of L, so every chunk has exactly L steps; the step loops then carry
+// no bounds tests, and when the x ring is one chunk deep (kBwdDepth == L) the slot of step
+// tt is tt and the step it prefetches is step tt of the next chunk (no ring walker).
+template <int K, int G, int PSI, typename XT, int L, int LAYOUT, bool BETA, bool FULL>
 __global__ void __launch_bounds__(bwd_threads(bwd_lane_compartments(K, G, xt_code<XT>(), L)),
                                   bwd_threads(bwd_lane_compartments(K, G, xt_code<XT>(), L)) == 128 ? 3 : 2)
 dendsn_backward_kernel(const BwdArgs A) {
@@ -1188,6 +1206,7 @@ dendsn_backward_kernel(const BwdArgs A) {
     // measured faster there
     constexpr bool BASYNC = DENDSN_BWD_ASYNC && SHIST && V::kAsync;
     constexpr int D = kBwdDepth;
+    constexpr bool SLOTS = FULL && BASYNC && D == L;
     const Geometry &g = A.g;
     const Params &P = A.p;
     const ThreadPos pos = thread_pos<LPN>(g);
@@ -1287,7 +1306,7 @@ dendsn_backward_kernel(const BwdArgs A) {
         float dvn = 0.f;              // dL/dV^s[t+1]
         for (int c = nc - 1; c >= 0; --c) {
             const int t0 = c * L;
-            const int ncur = min(L, T - t0);
+            const int ncur = FULL ? L : min(L, T - t0);
             // state entering the chunk: zero at t = 0, else the forward's checkpoint
             typename AR::St vd0;
             if (!MULTI || c == 0) {
@@ -1301,7 +1320,7 @@ dendsn_backward_kernel(const BwdArgs A) {
             const bool has_next = same_row || (i + 1 < pos.nrows);
             const int cn = same_row ? c - 1 : nc - 1;
             const int tn = cn * L;
-            const int nnext = has_next ? min(L, T - tn) : 0;
+            const int nnext = has_next ? (FULL ? L : min(L, T - tn)) : 0;
             const int64_t jn = same_row ? j : j + jstep;
             const XT *xn = (same_row ? xrow : xrow + rX) + (int64_t)tn * sX;
             const XT *gsn = (same_row ? gsrow : gsrow + jstep) + (int64_t)tn * BN;
@@ -1346,11 +1365,15 @@ dendsn_backward_kernel(const BwdArgs A) {
                     if (tt < ncur) {
                         if constexpr (BASYNC) {
                             cp_async_wait<D - 1>();
-                            V::unpack(xring[xslot * NT], xv);
+                            V::unpack(xring[(SLOTS ? tt : xslot) * NT], xv);
                         }
                         const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
-                        if constexpr (BASYNC) {
+                        if constexpr (SLOTS) {
                             // the slot's value has been used (z depends on it): refill it
+                            // with the same step of the next chunk
+                            if (has_next) V::copy_async(xring + tt * NT, xn + (int64_t)tt * sX, ks, z);
+                            cp_async_commit();
+                        } else if constexpr (BASYNC) {
                             if (wr < pos.nrows) V::copy_async(xring + xslot * NT, wp, ks, z);
                             cp_async_commit();
                             walk();
@@ -1436,7 +1459,7 @@ dendsn_backward_kernel(const BwdArgs A) {
     // (slot NA: beta, counted once per neuron, by its first lane)
     constexpr int NA1 = NA + 1;
     float v[NA1];
-    AR::acc_export(acc, v);
+    AR::acc_export(lp, acc, v);
     v[NA] = (BETA && pos.sub == 0) ? gbeta : 0.f;
 #pragma unroll
     for (int a = 0; a < NA1; ++a)
@@ -1531,16 +1554,23 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
     const size_t ring = (DENDSN_BWD_ASYNC && shist && XI::kAsync) ? xraw * kBwdDepth * NT : 0;
     const size_t smem = (red > hist + ring ? red : hist + ring) +
                         kappa_smem_bytes(a.p.mask_mode, KT / G, NT);
-    if (a.want_beta) {
-        cudaError_t e = allow_smem(dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, true>, smem);
+    auto go = [&](auto kernel) {
+        cudaError_t e = allow_smem(kernel, smem);
         if (e != cudaSuccess) return e;
-        dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, true><<<blocks, NT, smem, s>>>(a);
-    } else {
-        cudaError_t e = allow_smem(dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, false>, smem);
-        if (e != cudaSuccess) return e;
-        dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, false><<<blocks, NT, smem, s>>>(a);
+        kernel<<<blocks, NT, smem, s>>>(a);
+        return cudaGetLastError();
+    };
+    // full chunks: deeper conv layer 906 -> 738 us, event layer 1829 -> 1755 us; not for
+    // 4-step chunks of neurons split over lanes, whose full-chunk build spills in the loop
+    // (token layer 265 -> 314 us)
+    constexpr bool kFull = L == 8 || K / KT == 1;
+    if constexpr (kFull) {
+        if (a.g.T % L == 0)
+            return a.want_beta ? go(dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, true, true>)
+                               : go(dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, false, true>);
     }
-    return cudaGetLastError();
+    return a.want_beta ? go(dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, true, false>)
+                       : go(dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, false, false>);
 }
 
 }  // namespace dendsn
