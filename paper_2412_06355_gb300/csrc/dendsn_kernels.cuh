@@ -301,6 +301,7 @@ __host__ __device__ constexpr size_t kappa_smem_bytes(int mask_mode, int KTb, in
 // dL/dalpha, dL/dxi, dL/dzeta are scaled by 1/zeta once, in acc_export.
 template <int KT, int PSI, bool TREE>
 struct PairArith {
+    static constexpr bool kTree = TREE;
     static constexpr int N2 = KT / 2;
     static constexpr int KTb = KT;
     struct LP { float2 a[N2], nxi[N2], iz[N2], km[N2], lm[N2]; };
@@ -349,6 +350,20 @@ struct PairArith {
 #pragma unroll
         for (int m = 0; m < N2; ++m) s.v[m] = make_float2(v[2 * m], v[2 * m + 1]);
     }
+    // Pair m of one forward step (Eqs. methods-compartment, -branch-aggregation,
+    // -mexican-hat): advances its V^d by the input x2 and returns its branch outputs Y.
+    static __device__ __forceinline__ float2 pair_y(const LP &lp, int m, float2 &vd, float2 x2) {
+        vd = ffma2(lp.a[m], vd, x2);
+        const float2 u = ffma2(vd, lp.iz[m], lp.nxi[m]);
+        if constexpr (PSI == PSI_MEXHAT) {
+            const float2 ss = fmul2(u, u);
+            const float2 t = fmul2(f2(kNegHalfLog2e), ss);
+            const float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
+            return ffma2(neg2(ss), e, e);                        // (1 - r^2) e^{-r^2/2}
+        } else {
+            return make_float2(fabsf(u.x), fabsf(u.y));          // r
+        }
+    }
     // The lane's share of Z as one chain over the pairs (used when the forward and the
     // backward give a neuron the same lanes; see step for the tree order).
     static __device__ __forceinline__ float step_chain(const LP &lp, St &vd, const float (&x)[KT],
@@ -356,17 +371,7 @@ struct PairArith {
         float2 zp = f2(0.f);
 #pragma unroll
         for (int m = 0; m < N2; ++m) {
-            vd.v[m] = ffma2(lp.a[m], vd.v[m], make_float2(x[2 * m], x[2 * m + 1]));
-            const float2 u = ffma2(vd.v[m], lp.iz[m], lp.nxi[m]);
-            float2 y;
-            if constexpr (PSI == PSI_MEXHAT) {
-                const float2 ss = fmul2(u, u);
-                const float2 t = fmul2(f2(kNegHalfLog2e), ss);
-                const float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
-                y = ffma2(neg2(ss), e, e);                       // (1 - r^2) e^{-r^2/2}
-            } else {
-                y = make_float2(fabsf(u.x), fabsf(u.y));         // r
-            }
+            const float2 y = pair_y(lp, m, vd.v[m], make_float2(x[2 * m], x[2 * m + 1]));
             zp = (m == 0) ? fmul2(lp.km[m], y) : ffma2(lp.km[m], y, zp);
         }
         float z = __fadd_rn(zp.x, zp.y);
@@ -395,17 +400,7 @@ struct PairArith {
 #pragma unroll
             for (int h = 0; h < 2 && 2 * q + h < N2; ++h) {
                 const int m = 2 * q + h;
-                vd.v[m] = ffma2(lp.a[m], vd.v[m], make_float2(x[2 * m], x[2 * m + 1]));
-                const float2 u = ffma2(vd.v[m], lp.iz[m], lp.nxi[m]);
-                float2 y;
-                if constexpr (PSI == PSI_MEXHAT) {
-                    const float2 ss = fmul2(u, u);
-                    const float2 t = fmul2(f2(kNegHalfLog2e), ss);
-                    const float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
-                    y = ffma2(neg2(ss), e, e);                   // (1 - r^2) e^{-r^2/2}
-                } else {
-                    y = make_float2(fabsf(u.x), fabsf(u.y));     // r
-                }
+                const float2 y = pair_y(lp, m, vd.v[m], make_float2(x[2 * m], x[2 * m + 1]));
                 acc = (h == 0) ? fmul2(lp.km[m], y) : ffma2(lp.km[m], y, acc);
             }
             gv[q] = __fadd_rn(acc.x, acc.y);
@@ -448,7 +443,16 @@ struct PairArith {
         const float2 res2 = f2(res);
 #pragma unroll
         for (int m = 0; m < N2; ++m) {
-            const float2 u = ffma2(vdt.v[m], lp.iz[m], lp.nxi[m]);
+            const float2 g = pair_back(lp, m, vdt.v[m], vdp.v[m], dz2, res2, Ad.v[m], acc);
+            gx[2 * m] = g.x;
+            gx[2 * m + 1] = g.y;
+        }
+    }
+    // Pair m of one reverse step (see backward); returns dL/dX[t] of the pair.
+    static __device__ __forceinline__ float2 pair_back(const LP &lp, int m, float2 vdt, float2 vdp,
+                                                       float2 dz2, float2 res2, float2 &Adm, Acc &acc) {
+        {
+            const float2 u = ffma2(vdt, lp.iz[m], lp.nxi[m]);
             const float2 gy = fmul2(lp.km[m], dz2);              // dL/dY
             float2 y, du;                                        // m Y, dL/du
             if constexpr (PSI == PSI_MEXHAT) {
@@ -466,11 +470,9 @@ struct PairArith {
             acc.ngxi[m] = fadd2(acc.ngxi[m], du);                // zeta dxi = -sum du
             acc.ngz[m] = ffma2(u, du, acc.ngz[m]);               // zeta dzeta = -sum u du
             acc.gk[m] = ffma2(y, dz2, acc.gk[m]);                // dkappa = sum m Y dz
-            Ad.v[m] = ffma2(lp.a[m], Ad.v[m], du);
-            acc.ga[m] = ffma2(Ad.v[m], vdp.v[m], acc.ga[m]);     // zeta dalpha
-            const float2 g = ffma2(Ad.v[m], lp.iz[m], res2);
-            gx[2 * m] = g.x;
-            gx[2 * m + 1] = g.y;
+            Adm = ffma2(lp.a[m], Adm, du);
+            acc.ga[m] = ffma2(Adm, vdp, acc.ga[m]);              // zeta dalpha
+            return ffma2(Adm, lp.iz[m], res2);
         }
     }
 };
@@ -743,6 +745,9 @@ template <typename XT, typename Raw> constexpr int fwd_depth() {
 #define DENDSN_BWD_ASYNC 1
 #endif
 constexpr int kBwdDepth = 8;   // steps of x in flight per thread in the backward's cp.async ring
+#ifndef DENDSN_BWD_PHASED
+#define DENDSN_BWD_PHASED 1
+#endif
 
 // Asynchronous 4/8/16-byte global -> shared copy (PTX cp.async). `dep` is an unused
 // operand that orders the copy after the computation producing it.
@@ -1173,6 +1178,56 @@ dendsn_forward_staged_kernel(const FwdArgs A) {
 }
 
 // ---------------------------------------------------------------- backward
+// Per-channel partial sums of a block's parameter-gradient vectors v (one per thread,
+// [alpha KT | xi KT | zeta KTb | kappa KTb | beta]) in a fixed order: segmented warp
+// shuffles over the columns of one channel, then the run leaders in shared memory (red,
+// NA1 * NT floats), one partial per (block, channel) to `partials`.
+template <int KT, int G, int LPN, int NT, int NA1>
+__device__ __forceinline__ void block_partials(const Geometry &g, const ThreadPos &pos,
+                                               float (&v)[NA1], float *red, float *partials) {
+    constexpr int KTb = KT / G;
+    constexpr int NA = NA1 - 1;
+    // stage 1: within a warp, columns of one channel come in aligned runs of g.seg
+    for (int d = 1; d < g.seg; d <<= 1) {
+#pragma unroll
+        for (int a = 0; a < NA1; ++a)
+            v[a] = __fadd_rn(v[a], __shfl_xor_sync(0xffffffffu, v[a], d * LPN));
+    }
+    // stage 2: run leaders meet in shared memory; red[a][tid] (reuses the history space)
+    __syncthreads();
+#pragma unroll
+    for (int a = 0; a < NA1; ++a) red[a * NT + threadIdx.x] = v[a];
+    __syncthreads();
+    const int ct = blockIdx.x % g.nCT;
+    const int p0 = ct * g.TXn;
+    const int p1 = min(p0 + g.TXn, g.P);            // exclusive
+    const int c_lo = p0 / g.inner;
+    const int nch = (p1 - 1) / g.inner - c_lo + 1;
+    const int NP = 2 * g.K + 2 * g.Kb + 1;          // per-channel gradient vector
+    float *out = partials + (int64_t)blockIdx.x * g.nch_max * NP;
+    const int items = nch * LPN * NA1;
+    for (int w = threadIdx.x; w < items; w += NT) {
+        const int a = w % NA1;
+        const int sub = (w / NA1) % LPN;
+        const int lc = w / (NA1 * LPN);
+        if (a == NA && sub > 0) continue;          // beta: one lane per neuron
+        const int c = c_lo + lc;
+        const int cx_lo = max(c * g.inner, p0) - p0;
+        const int cx_hi = min((c + 1) * g.inner, p1) - p0;
+        float sum = 0.f;
+        for (int ry = 0; ry < g.TY; ++ry)
+            for (int cx = cx_lo; cx < cx_hi; cx += g.seg)
+                sum = __fadd_rn(sum, red[a * NT + (ry * g.TXn + cx) * LPN + sub]);
+        int slot;
+        if (a < KT) slot = sub * KT + a;                                        // alpha
+        else if (a < 2 * KT) slot = g.K + sub * KT + (a - KT);                  // xi
+        else if (a < 2 * KT + KTb) slot = 2 * g.K + sub * KTb + (a - 2 * KT);   // zeta
+        else if (a < NA) slot = 2 * g.K + g.Kb + sub * KTb + (a - 2 * KT - KTb); // kappa
+        else slot = NP - 1;                                                     // beta
+        out[lc * NP + slot] = sum;
+    }
+}
+
 template <int KT, int G>
 constexpr int acc_count() { return 2 * KT + 2 * (KT / G); }
 
@@ -1464,47 +1519,177 @@ dendsn_backward_kernel(const BwdArgs A) {
 #pragma unroll
     for (int a = 0; a < NA1; ++a)
         if (!pos.active || (a < KT && P.stateless)) v[a] = 0.f;
-    // stage 1: within a warp, columns of one channel come in aligned runs of g.seg
-    for (int d = 1; d < g.seg; d <<= 1) {
-#pragma unroll
-        for (int a = 0; a < NA1; ++a)
-            v[a] = __fadd_rn(v[a], __shfl_xor_sync(0xffffffffu, v[a], d * LPN));
-    }
-    // stage 2: run leaders meet in shared memory; red[a][tid] (reuses the history space)
-    float *red = reinterpret_cast<float *>(sregion);
     if constexpr (BASYNC) cp_async_wait<0>();
-    __syncthreads();
+    block_partials<KT, G, LPN, NT>(g, pos, v, reinterpret_cast<float *>(sregion), A.partials);
+}
+
+// ---------------------------------------------------------------- phased backward
+// The backward for rows that are one full chunk (T == L) of neurons served whole by one
+// lane of 8 compartments (paired engine, G = 1, compartments innermost, no residual term;
+// the deeper bf16 conv layer). dendsn_backward_kernel walks each reverse step over all of
+// a lane's compartment pairs at once, so the adjoints, temporaries and history of every
+// pair are live together; here a row runs in phases so that the reverse scan holds one
+// pair at a time:
+//   1. recompute the chunk step by step (the forward's own step function, so Z and the
+//      spikes are bit-identical), writing V^d of every step and pair to shared memory;
+//      then fetch the next row's x into the freed ring;
+//   2. the soma in registers: V^s forward, then its reverse recursion for dL/dZ[t]
+//      (Eqs. methods-lif-reset-charge, methods-lif-fire, methods-sg);
+//   3. pair by pair, the dendritic reverse scan over the chunk (the same per-pair step as
+//      dendsn_backward_kernel); dL/dX[t] of a pair overwrites its V^d[t] slot, which the
+//      scan no longer needs;
+//   4. gather each step's dL/dX from shared memory and store it as one vector.
+// Every accumulator sees its terms in the same order as in dendsn_backward_kernel, so
+// the two kernels give bit-identical results.
+template <int K, int PSI, typename XT, int L, bool BETA>
+__global__ void __launch_bounds__(bwd_threads(K), bwd_threads(K) == 128 ? 3 : 2)
+dendsn_backward_phased_kernel(const BwdArgs A) {
+    constexpr int KT = K;
+    constexpr int NT = bwd_threads(KT);
+    constexpr int N2 = KT / 2;
+    constexpr int NA = acc_count<KT, 1>();
+    using V = XIO<XT, KT, 0>;
+    using S1 = Scalar<XT>;
+    using AR = Arith<KT, 1, PSI, XT>;
+    using XRaw = typename V::Raw;
+    static_assert(KT % 2 == 0 && AR::KTb == KT, "paired engine only");
+    const Geometry &g = A.g;
+    const Params &P = A.p;
+    const ThreadPos pos = thread_pos<1>(g);
+    typename AR::LP lp;
+    AR::load(P, g, pos.chan, 0, lp);
+    const int64_t sX = g.BN * K;
+    const int64_t BN = g.BN;
+    const int64_t j0 = pos.row0 * g.P + pos.p;
+    const int64_t jstep = (int64_t)pos.rstride * g.P;
+    const int64_t rX = jstep * K;
+    const XT *__restrict__ xrow = static_cast<const XT *>(A.x) + j0 * K;
+    const XT *__restrict__ gsrow = static_cast<const XT *>(A.gs) + j0;
+    XT *__restrict__ gxrow = static_cast<XT *>(A.gx) + j0 * K;
+    const float *gvrow = A.gv ? A.gv + j0 : nullptr;
+    const float kv = (P.detach || P.soft) ? 0.f : -P.beta;
+    const float cs = (P.detach || !P.soft) ? 0.f : -P.beta * P.theta;
+    const float b_spike = P.soft ? P.beta : 0.f;
+    const bool has_gv = A.gv != nullptr;
+
+    // dynamic shared memory: the lanes' kappa (per-neuron masks only), then the history
+    // [L][N2][NT] float2 and the x ring [L][NT], or (at the end) the reduction
+    extern __shared__ float4 smem_f4[];
+    char *const sregion = reinterpret_cast<char *>(smem_f4) + kappa_smem_bytes(P.mask_mode, KT, NT);
+    float2 *const hist = reinterpret_cast<float2 *>(sregion) + threadIdx.x;
+    XRaw *const xring = reinterpret_cast<XRaw *>(reinterpret_cast<float2 *>(sregion) + L * N2 * NT) +
+                        threadIdx.x;
+    if (pos.nrows > 0) {
 #pragma unroll
-    for (int a = 0; a < NA1; ++a) red[a * NT + threadIdx.x] = v[a];
-    __syncthreads();
-    const int ct = blockIdx.x % g.nCT;
-    const int p0 = ct * g.TXn;
-    const int p1 = min(p0 + g.TXn, g.P);            // exclusive
-    const int c_lo = p0 / g.inner;
-    const int nch = (p1 - 1) / g.inner - c_lo + 1;
-    const int NP = 2 * g.K + 2 * g.Kb + 1;          // per-channel gradient vector
-    float *out = A.partials + (int64_t)blockIdx.x * g.nch_max * NP;
-    const int items = nch * LPN * NA1;
-    for (int w = threadIdx.x; w < items; w += NT) {
-        const int a = w % NA1;
-        const int sub = (w / NA1) % LPN;
-        const int lc = w / (NA1 * LPN);
-        if (a == NA && sub > 0) continue;          // beta: one lane per neuron
-        const int c = c_lo + lc;
-        const int cx_lo = max(c * g.inner, p0) - p0;
-        const int cx_hi = min((c + 1) * g.inner, p1) - p0;
-        float sum = 0.f;
-        for (int ry = 0; ry < g.TY; ++ry)
-            for (int cx = cx_lo; cx < cx_hi; cx += g.seg)
-                sum = __fadd_rn(sum, red[a * NT + (ry * g.TXn + cx) * LPN + sub]);
-        int slot;
-        if (a < KT) slot = sub * KT + a;                                        // alpha
-        else if (a < 2 * KT) slot = g.K + sub * KT + (a - KT);                  // xi
-        else if (a < 2 * KT + KTb) slot = 2 * g.K + sub * KTb + (a - 2 * KT);   // zeta
-        else if (a < NA) slot = 2 * g.K + g.Kb + sub * KTb + (a - 2 * KT - KTb); // kappa
-        else slot = NP - 1;                                                     // beta
-        out[lc * NP + slot] = sum;
+        for (int tt = 0; tt < L; ++tt) V::copy_async(xring + tt * NT, xrow + (int64_t)tt * sX, 1, 0.f);
     }
+    cp_async_commit();
+
+    typename AR::Acc acc;
+    AR::acc_zero(acc);
+    float gbeta = 0.f;
+    MaskAhead<AR, NT> mask;
+    mask.init(P, g, j0, jstep, pos.chan, 0, pos.nrows, smem_f4);
+    for (int i = 0; i < pos.nrows; ++i) {
+        mask.advance(P, g, 0, i + 1 < pos.nrows, lp);
+        typename S1::Raw gsr[L];                 // grad_spikes of the row, used in phase 2
+#pragma unroll
+        for (int tt = 0; tt < L; ++tt) gsr[tt] = S1::load(gsrow + (int64_t)tt * BN);
+
+        // phase 1: recompute
+        cp_async_wait<0>();
+        float z[L];
+        {
+            typename AR::St vd;
+            AR::zero(vd);
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) {
+                float xv[KT];
+                V::unpack(xring[tt * NT], xv);
+                z[tt] = AR::step(lp, vd, xv, false, 0.f);
+#pragma unroll
+                for (int m = 0; m < N2; ++m) hist[(tt * N2 + m) * NT] = vd.v[m];
+            }
+        }
+        if (i + 1 < pos.nrows) {
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt)
+                V::copy_async(xring + tt * NT, xrow + rX + (int64_t)tt * sX, 1, z[L - 1]);
+        }
+        cp_async_commit();
+
+        // phase 2: the soma forward, then dL/dV^s backwards in time (dL/dZ = dL/dV^s)
+        float dz[L];
+        {
+            float v = 0.f;
+            bool s = false;
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) {
+                v = soma_charge(z[tt], v, s, P);
+                s = v >= P.theta;
+                z[tt] = v;                       // z now holds V^s
+            }
+            float dvn = 0.f;                     // dL/dV^s[t+1]
+#pragma unroll
+            for (int tt = L - 1; tt >= 0; --tt) {
+                const float vs = z[tt];
+                const bool st = vs >= P.theta;
+                if constexpr (BETA) {
+                    const float leak = st ? (P.soft ? __fsub_rn(vs, P.theta) : 0.f) : vs;
+                    gbeta = __fmaf_rn(dvn, leak, gbeta);
+                }
+                const float dvds = __fmaf_rn(kv, vs, cs);
+                const float dvdv = st ? b_spike : P.beta;
+                const float ds = __fmaf_rn(dvds, dvn, S1::unpack(gsr[tt]));
+                float dv = __fmaf_rn(surrogate(__fsub_rn(vs, P.theta)), ds, __fmul_rn(dvdv, dvn));
+                if (has_gv) dv = __fadd_rn(dv, __ldcs(gvrow + (int64_t)tt * BN));
+                dz[tt] = dv;
+                dvn = dv;
+            }
+        }
+
+        // phase 3: the dendritic reverse scan, one pair at a time
+#pragma unroll
+        for (int m = 0; m < N2; ++m) {
+            float2 Ad = f2(0.f);
+            float2 vdt = hist[((L - 1) * N2 + m) * NT];
+#pragma unroll
+            for (int tt = L - 1; tt >= 0; --tt) {
+                const float2 vdp = tt > 0 ? hist[((tt > 0 ? tt - 1 : 0) * N2 + m) * NT] : f2(0.f);
+                hist[(tt * N2 + m) * NT] = AR::pair_back(lp, m, vdt, vdp, f2(dz[tt]), f2(0.f), Ad, acc);
+                vdt = vdp;
+            }
+        }
+
+        // phase 4: dL/dX of each step as one vector
+        if (pos.active) {
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) {
+                float gxv[KT];
+#pragma unroll
+                for (int m = 0; m < N2; ++m) {
+                    const float2 q = hist[(tt * N2 + m) * NT];
+                    gxv[2 * m] = q.x;
+                    gxv[2 * m + 1] = q.y;
+                }
+                V::store(gxrow + (int64_t)tt * sX, 1, gxv);
+            }
+        }
+        xrow += rX;
+        gsrow += jstep;
+        gxrow += rX;
+        if (has_gv) gvrow += jstep;
+    }
+
+    constexpr int NA1 = NA + 1;
+    float v[NA1];
+    AR::acc_export(lp, acc, v);
+    v[NA] = BETA ? gbeta : 0.f;
+#pragma unroll
+    for (int a = 0; a < NA1; ++a)
+        if (!pos.active || (a < KT && P.stateless)) v[a] = 0.f;
+    cp_async_wait<0>();
+    block_partials<KT, 1, 1, NT>(g, pos, v, reinterpret_cast<float *>(sregion), A.partials);
 }
 
 // ---------------------------------------------------------------- launchers
@@ -1554,12 +1739,24 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
     const size_t ring = (DENDSN_BWD_ASYNC && shist && XI::kAsync) ? xraw * kBwdDepth * NT : 0;
     const size_t smem = (red > hist + ring ? red : hist + ring) +
                         kappa_smem_bytes(a.p.mask_mode, KT / G, NT);
-    auto go = [&](auto kernel) {
-        cudaError_t e = allow_smem(kernel, smem);
+    auto go_smem = [&](auto kernel, size_t bytes) {
+        cudaError_t e = allow_smem(kernel, bytes);
         if (e != cudaSuccess) return e;
-        kernel<<<blocks, NT, smem, s>>>(a);
+        kernel<<<blocks, NT, bytes, s>>>(a);
         return cudaGetLastError();
     };
+    auto go = [&](auto kernel) { return go_smem(kernel, smem); };
+    // rows of one full chunk, a whole 8-compartment neuron per lane: the phased kernel
+    constexpr bool kPhased = DENDSN_BWD_PHASED && LAYOUT == 0 && G == 1 && K == 8 && KT == K &&
+                             XI::kAsync;
+    if constexpr (kPhased) {
+        if (a.g.T == L && !a.p.residual) {
+            const size_t ph = sizeof(float) * KT * L * NT + xraw * L * NT;
+            const size_t psm = (red > ph ? red : ph) + kappa_smem_bytes(a.p.mask_mode, KT, NT);
+            return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true>, psm)
+                               : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false>, psm);
+        }
+    }
     // full chunks: deeper conv layer 906 -> 738 us, event layer 1829 -> 1755 us; not for
     // 4-step chunks of neurons split over lanes, whose full-chunk build spills in the loop
     // (token layer 265 -> 314 us)

@@ -72,8 +72,8 @@ def test_every_compiled_kg(K, G, layout):
 
 @pytest.mark.parametrize("inner", [40, 64])      # 64: the forward stages inputs per warp
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-@pytest.mark.parametrize("K,G,T", [(2, 2, 3), (4, 2, 4), (4, 1, 12), (8, 1, 4), (8, 2, 9),
-                                   (16, 4, 5)])
+@pytest.mark.parametrize("K,G,T", [(2, 2, 3), (4, 2, 4), (4, 1, 12), (8, 1, 4), (8, 1, 8),
+                                   (8, 2, 9), (16, 4, 5)])
 def test_paper_layout_is_bitwise_the_kinner_layer(K, G, T, dtype, inner):
     """Only the addresses differ between the layouts: every output must be bit-identical."""
     w = workloads.Workload("lay", T=T, B=3, N=4 * 2 * inner, K=K, G=G, C=4, inner=inner,
@@ -108,6 +108,19 @@ def test_paper_layout_is_bitwise_the_kinner_layer(K, G, T, dtype, inner):
 def test_variants(kw):
     w = workloads.Workload("var", T=6, B=4, N=4 * 96, K=8, G=1, C=4, inner=96, dtype="f32",
                            psi="mh", reset="hard", seed=7).with_(**kw)
+    check_layer(w)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("kw", [
+    dict(), dict(mask_p=0.5, mask_per_neuron=True), dict(reset="soft", psi="identity"),
+    dict(detach_reset=True), dict(stateless=True), dict(residual=True), dict(T=4),
+], ids=lambda kw: "-".join(f"{k}={v}" for k, v in kw.items()) or "plain")
+def test_one_chunk_rows_of_whole_neurons(kw, dtype):
+    # T == 8 (or 4): rows of one full chunk, 8 compartments per lane -- the phased backward
+    # (the residual variant takes the chunked kernel)
+    w = workloads.Workload("phased", T=8, B=5, N=3 * 128, K=8, G=1, C=3, inner=128,
+                           dtype=dtype, psi="mh", reset="hard", seed=41).with_(**kw)
     check_layer(w)
 
 
