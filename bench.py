@@ -139,6 +139,25 @@ class ClockSampler:
                 "samples": len(win), "note": note}
 
 
+# ------------------------------------------------------------------ kernel names
+def kernel_names(w):
+    """(forward, backward) kernels the library launches for workload w, following its plan:
+    narrow long-horizon layers take the time-parallel kernels; rows of one full chunk
+    (T = 4 or 8) whose 8 compartments sit on one lane, compartments innermost and no
+    residual term, take the phased backward (one lane per neuron: bf16, or float32 with
+    8-step chunks); the rest the chunked kernels."""
+    if w.T >= 256 and w.B * w.N <= 2048:
+        return "tp_forward_kernel", "tp_backward_kernel"
+    L = 4 if w.T <= 4 else 8
+    layout0 = w.layout == "kinner" or w.K == 1 or w.inner == 1
+    staged = (not layout0 and 2 <= w.K <= 8 and w.inner % 32 == 0)
+    fwd = "dendsn_forward_staged_kernel" if staged else "dendsn_forward_kernel"
+    one_lane = w.K == 8 and w.G == 1 and (w.dtype == "bf16" or L == 8)
+    if one_lane and layout0 and w.T == L and not w.residual:
+        return fwd, "dendsn_backward_phased_kernel"
+    return fwd, "dendsn_backward_kernel"
+
+
 # ------------------------------------------------------------------ traffic record
 def _strip_comments(src: str) -> str:
     """C/C++ source without // and /* */ comments and blank lines (comments do not change
@@ -550,10 +569,11 @@ def run_ours(args):
     ops = w.fp32_ops_per_neuron_step()
     fwd_avg, bwd_avg = statistics.mean(fwd_ms), statistics.mean(bwd_ms)
     peak, peak_kind = measured_hbm_peak()
+    fname, bname = kernel_names(w)
     if bwd_avg >= fwd_avg:
-        kname, kbytes, kms, kops = "dendsn_backward_kernel", ab["backward"], bwd_avg, ops["backward"]
+        kname, kbytes, kms, kops = bname, ab["backward"], bwd_avg, ops["backward"]
     else:
-        kname, kbytes, kms, kops = "dendsn_forward_kernel", ab["forward"], fwd_avg, ops["forward"]
+        kname, kbytes, kms, kops = fname, ab["forward"], fwd_avg, ops["forward"]
     achieved = kbytes / (kms / 1e3) / 1e9
     # the float32 roof of the same kernel: its float32 operations (a cost model counted from
     # the equations) against SMs x 128 FMA lanes x the SM clock

@@ -1757,10 +1757,12 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
                                : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false>, psm);
         }
     }
-    // full chunks: deeper conv layer 906 -> 738 us, event layer 1829 -> 1755 us; not for
-    // 4-step chunks of neurons split over lanes, whose full-chunk build spills in the loop
-    // (token layer 265 -> 314 us)
-    constexpr bool kFull = L == 8 || K / KT == 1;
+    // full chunks: deeper conv layer 906 -> 738 us, event layer 1829 -> 1755 us, conv layer
+    // 219.7 -> 217 us; with 4-step chunks only for whole neurons on one lane, one compartment
+    // per branch and compartments innermost: the other 4-step full-chunk builds spill in
+    // the loop (token layer 265 -> 314 us, conv layer in the paper layout with two
+    // compartments per branch 232 -> 242 us)
+    constexpr bool kFull = L == 8 || (K / KT == 1 && G == 1 && LAYOUT == 0);
     if constexpr (kFull) {
         if (a.g.T % L == 0)
             return a.want_beta ? go(dendsn_backward_kernel<K, G, PSI, T, L, LAYOUT, true, true>)
