@@ -26,7 +26,12 @@
 // grad_x. Parameter-gradient partials stay in registers per thread, are reduced per
 // channel inside the block in a fixed order (segmented warp shuffles, then shared
 // memory), written to scratch, and summed over blocks in a fixed order by a
-// finalize kernel: the parameter gradients are deterministic.
+// finalize kernel: the parameter gradients are deterministic. When T is a multiple
+// of L a full-chunk build of the same kernel drops the step bounds tests. Rows of
+// one full chunk of whole 8-compartment neurons take dendsn_backward_phased_kernel,
+// which runs a row in phases (recompute into shared memory, soma in registers,
+// dendritic reverse scan one compartment pair at a time) and gives bit-identical
+// results with fewer live registers.
 //
 // Arithmetic. With one compartment per branch (G = 1) the per-compartment work is
 // done two compartments at a time with the paired fp32 instructions of sm_100+
