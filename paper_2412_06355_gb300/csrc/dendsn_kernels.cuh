@@ -914,9 +914,12 @@ dendsn_forward_kernel(const FwdArgs A) {
         // The step loop is specialised on whether V^s and checkpoints are written and on
         // whether T divides the ring depth (then the step fetched D steps ahead is the
         // same step D/T rows further on: no walker needed).
-        auto rows = [&](auto extra, auto div) {
-            // EXTRA: V^s output and/or checkpoints requested (each still tested inside)
+        auto rows = [&](auto extra, auto div, auto tc) {
+            // EXTRA: V^s output and/or checkpoints requested (each still tested inside);
+            // TC > 0: T == TC known at compile time (the step loop unrolls; slots are the
+            // row's first slot plus the step)
             constexpr bool EXTRA = decltype(extra)::value, DIV = decltype(div)::value;
+            constexpr int TC = decltype(tc)::value;
             int slot = 0;
             int64_t j = j0;
             const int rows_ahead = DIV ? D / T : 0;
@@ -936,17 +939,17 @@ dendsn_forward_kernel(const FwdArgs A) {
                 float *vp = vr;
                 const XT *cp = xr;                       // this step's x in global memory
                 const bool fetch_row = i + rows_ahead < pos.nrows;
-                for (int t = 0; t < T; ++t) {
+                auto step = [&](int t, int sl) {
                     cp_async_wait<D - 1>();
                     float xv[KT];
-                    V::unpack(ring[slot * NT], xv);
+                    V::unpack(ring[sl * NT], xv);
                     const float z = soma_input<AR, KT, LPN>(lp, vd, xv, residual, inv_k);
                     // the slot's value has been used (z depends on it): refill it
                     if constexpr (DIV) {
-                        if (fetch_row) V::copy_async(ring + slot * NT, cp + ahead, ks, z);
+                        if (fetch_row) V::copy_async(ring + sl * NT, cp + ahead, ks, z);
                         cp += sX;
                     } else {
-                        if (ir < pos.nrows) V::copy_async(ring + slot * NT, ip, ks, z);
+                        if (ir < pos.nrows) V::copy_async(ring + sl * NT, ip, ks, z);
                         ip += sX;
                         if (++it == T) { it = 0; ++ir; ip += row_jump; }
                     }
@@ -970,7 +973,16 @@ dendsn_forward_kernel(const FwdArgs A) {
                             if (pos.sub == 0) __stcs(A.ck_vs + (int64_t)ck * BN + j, v);
                         }
                     }
-                    slot = (slot == D - 1) ? 0 : slot + 1;
+                };
+                if constexpr (TC > 0) {
+#pragma unroll
+                    for (int t = 0; t < TC; ++t) step(t, slot + t);
+                    slot = (slot + TC == D) ? 0 : slot + TC;
+                } else {
+                    for (int t = 0; t < T; ++t) {
+                        step(t, slot);
+                        slot = (slot == D - 1) ? 0 : slot + 1;
+                    }
                 }
                 xr += rX;
                 sr += jstep;
@@ -982,11 +994,16 @@ dendsn_forward_kernel(const FwdArgs A) {
         };
         using yes = std::true_type;
         using no = std::false_type;
+        using tc0 = std::integral_constant<int, 0>;
         const bool div = (D % T) == 0;
         if (vrow != nullptr || write_ck) {
-            if (div) rows(yes{}, yes{}); else rows(yes{}, no{});
+            if (div) rows(yes{}, yes{}, tc0{}); else rows(yes{}, no{}, tc0{});
+        } else if (div) {
+            if (T == 4) rows(no{}, yes{}, std::integral_constant<int, 4>{});
+            else if (T == 8) rows(no{}, yes{}, std::integral_constant<int, 8>{});
+            else rows(no{}, yes{}, tc0{});
         } else {
-            if (div) rows(no{}, yes{}); else rows(no{}, no{});
+            rows(no{}, no{}, tc0{});
         }
         cp_async_wait<0>();
         return;
