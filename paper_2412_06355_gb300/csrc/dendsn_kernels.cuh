@@ -1769,6 +1769,8 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
     };
     auto go = [&](auto kernel) { return go_smem(kernel, smem); };
     // rows of one full chunk, a whole 8-compartment neuron per lane: the phased kernel
+    // (deeper conv layer 738 -> 556 us; for the 4-compartment conv layer and for the token
+    // layer on one 8-compartment lane it measured slower: 217 -> 280 us, 261 -> 295 us)
     constexpr bool kPhased = DENDSN_BWD_PHASED && LAYOUT == 0 && G == 1 && K == 8 && KT == K &&
                              XI::kAsync;
     if constexpr (kPhased) {
@@ -1783,7 +1785,7 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
     // 219.7 -> 217 us; with 4-step chunks only for whole neurons on one lane, one compartment
     // per branch and compartments innermost: the other 4-step full-chunk builds spill in
     // the loop (token layer 265 -> 314 us, conv layer in the paper layout with two
-    // compartments per branch 232 -> 242 us)
+    // compartments per branch 230 -> 240 us)
     constexpr bool kFull = L == 8 || (K / KT == 1 && G == 1 && LAYOUT == 0);
     if constexpr (kFull) {
         if (a.g.T % L == 0)
