@@ -31,7 +31,9 @@
 // one full chunk of whole 8-compartment neurons take dendsn_backward_phased_kernel,
 // which runs a row in phases (recompute into shared memory, soma in registers,
 // dendritic reverse scan one compartment pair at a time) and gives bit-identical
-// results with fewer live registers.
+// results with fewer live registers. 4-step rows of 8-compartment float32 neurons on
+// two lanes take dendsn_backward_rowpair_kernel: the same phases over two rows per
+// thread, each paired instruction carrying one compartment of both rows.
 //
 // Arithmetic. With one compartment per branch (G = 1) the per-compartment work is
 // done two compartments at a time with the paired fp32 instructions of sm_100+
@@ -752,6 +754,9 @@ template <typename XT, typename Raw> constexpr int fwd_depth() {
 constexpr int kBwdDepth = 8;   // steps of x in flight per thread in the backward's cp.async ring
 #ifndef DENDSN_BWD_PHASED
 #define DENDSN_BWD_PHASED 1
+#endif
+#ifndef DENDSN_BWD_ROWPAIR
+#define DENDSN_BWD_ROWPAIR 1
 #endif
 
 // Asynchronous 4/8/16-byte global -> shared copy (PTX cp.async). `dep` is an unused
@@ -1714,6 +1719,282 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
     block_partials<KT, 1, 1, NT>(g, pos, v, reinterpret_cast<float *>(sregion), A.partials);
 }
 
+// ---------------------------------------------------------------- row-pair backward
+// The backward for 4-step rows (T == 4) of 8-compartment float32 neurons served by two
+// lanes of four compartments (the transformer-token layer; no residual term). Each thread
+// takes its half-neuron of two of its rows at once: a paired instruction carries the same
+// compartment of the two neurons (both in the same column, so with the same parameters),
+// and the soma recursions and the per-row bookkeeping are shared by the two rows. A row
+// pair runs in the phases of dendsn_backward_phased_kernel:
+//   1. recompute (Z of each row in the paired engine's tree order and the same lane
+//      butterfly, so Z and the spikes are bit-identical to the forward's), V^d of every
+//      step and compartment to shared memory; then x of the next row pair is requested;
+//   2. the two somas forward, then their reverse recursions, in paired registers; then the
+//      next pair's dL/dS (and per-neuron mask bytes) are requested;
+//   3. the dendritic reverse scan one compartment at a time, dL/dX overwriting V^d[t];
+//   4. each step's dL/dX of each row gathered and stored as one vector.
+// x, dL/dS and the mask bytes of a row pair arrive by cp.async one pair ahead. A thread
+// with an odd number of rows pairs its last row with a copy of itself whose dL/dS and
+// dL/dV^s are zero (its contributions are exactly zero) and whose dL/dX is not stored.
+template <int PSI, int LAYOUT, bool BETA>
+__global__ void __launch_bounds__(256, 2)
+dendsn_backward_rowpair_kernel(const BwdArgs A) {
+    constexpr int K = 8, KT = 4, LPN = 2, L = 4, NT = 256;
+    constexpr int NA = acc_count<KT, 1>();
+    using V = XIO<float, KT, LAYOUT>;
+    using XRaw = typename V::Raw;
+    static_assert(bwd_threads(KT) == NT, "the plan tiles this backward with bwd_threads(4)");
+    const Geometry &g = A.g;
+    const Params &P = A.p;
+    const ThreadPos pos = thread_pos<LPN>(g);
+    // the lane's compartments: alpha, -xi/zeta, 1/zeta, kappa * m (per channel) and m
+    float a[KT], nxi[KT], iz[KT], kmc[KT], mkc[KT];
+    load_param_arrays<KT, 1>(P, g, pos.chan, pos.sub, a, nxi, iz, kmc, mkc);
+    const int64_t sX = g.BN * K;
+    const int64_t BN = g.BN;
+    const int64_t j0 = pos.row0 * g.P + pos.p;
+    const int64_t jstep = (int64_t)pos.rstride * g.P;
+    const int64_t rX = jstep * K;
+    const int64_t ks = LAYOUT == 0 ? 1 : g.inner;
+    const int64_t xoff = lane_x_offset<LAYOUT>(j0, pos.sub, KT, K, g.inner);
+    const float *const x0 = static_cast<const float *>(A.x) + xoff;
+    const float *const gs0 = static_cast<const float *>(A.gs) + j0;
+    float *const gx0 = static_cast<float *>(A.gx) + xoff;
+    const float kv = (P.detach || P.soft) ? 0.f : -P.beta;
+    const float cs = (P.detach || !P.soft) ? 0.f : -P.beta * P.theta;
+    const float b_spike = P.soft ? P.beta : 0.f;
+    const bool has_gv = A.gv != nullptr;
+    const int nrows = pos.nrows;
+    const int nq = (nrows + 1) / 2;              // row pairs
+
+    // dynamic shared memory: history [L][KT][NT] float2, x [2][L][NT], dL/dS [2][L][NT],
+    // mask bytes [2][NT]; or (at the end) the reduction
+    extern __shared__ float4 smem_f4[];
+    char *const sregion = reinterpret_cast<char *>(smem_f4);
+    float2 *const hist = reinterpret_cast<float2 *>(sregion) + threadIdx.x;
+    XRaw *const xring = reinterpret_cast<XRaw *>(sregion + sizeof(float2) * L * KT * NT) + threadIdx.x;
+    float *const gring = reinterpret_cast<float *>(sregion + sizeof(float2) * L * KT * NT +
+                                                   sizeof(XRaw) * 2 * L * NT) + threadIdx.x;
+    uint32_t *const mring = reinterpret_cast<uint32_t *>(sregion + sizeof(float2) * L * KT * NT +
+                                                         sizeof(XRaw) * 2 * L * NT +
+                                                         sizeof(float) * 2 * L * NT) + threadIdx.x;
+    // neuron (within a sample) of the first row of the pair being fetched, for the masks
+    const int nstep = (int)(jstep % g.N);
+    int nf = (int)(j0 % g.N);
+    auto fetch_x = [&](int q, float dep) {
+        const int k = 2 * q;
+        if (k < nrows) {
+            const float *p1 = x0 + (int64_t)k * rX;
+            const float *p2 = (k + 1 < nrows) ? p1 + rX : p1;
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) {
+                V::copy_async(xring + tt * NT, p1 + (int64_t)tt * sX, ks, dep);
+                V::copy_async(xring + (L + tt) * NT, p2 + (int64_t)tt * sX, ks, dep);
+            }
+        }
+        cp_async_commit();
+    };
+    auto fetch_gs = [&](int q, float dep) {
+        const int k = 2 * q;
+        if (k < nrows) {
+            const bool two = k + 1 < nrows;
+            const float *p1 = gs0 + (int64_t)k * jstep;
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) {
+                cp_async<4>(gring + tt * NT, p1 + (int64_t)tt * BN, dep);
+                if (two) cp_async<4>(gring + (L + tt) * NT, p1 + jstep + (int64_t)tt * BN, dep);
+                else gring[(L + tt) * NT] = 0.f;
+            }
+            if (P.mask_mode == 2) {
+                int n2 = nf + nstep;
+                if (n2 >= g.N) n2 -= g.N;
+                cp_async<4>(mring, P.mask + (int64_t)nf * g.Kb + pos.sub * KT, dep);
+                cp_async<4>(mring + NT, P.mask + (int64_t)(two ? n2 : nf) * g.Kb + pos.sub * KT, dep);
+                nf = n2 + nstep;
+                if (nf >= g.N) nf -= g.N;
+            }
+        }
+        cp_async_commit();
+    };
+    fetch_x(0, 0.f);
+    fetch_gs(0, 0.f);
+
+    float2 ga[KT], ngxi[KT], ngz[KT], gk[KT];
+#pragma unroll
+    for (int c = 0; c < KT; ++c) { ga[c] = f2(0.f); ngxi[c] = f2(0.f); ngz[c] = f2(0.f); gk[c] = f2(0.f); }
+    float2 gb = f2(0.f);
+    for (int q = 0; q < nq; ++q) {
+        const int k = 2 * q;
+        const bool two = k + 1 < nrows;
+        cp_async_wait<0>();
+        // the two rows' kappa * m and mask terms (exponent 0 / -inf, or m for the identity)
+        float2 km2[KT], lm2[KT];
+        if (P.mask_mode == 2) {
+            const uint32_t m1 = mring[0], m2 = mring[NT];
+#pragma unroll
+            for (int c = 0; c < KT; ++c) {
+                const bool on1 = ((m1 >> (8 * c)) & 0xffu) != 0u, on2 = ((m2 >> (8 * c)) & 0xffu) != 0u;
+                km2[c] = make_float2(on1 ? kmc[c] : 0.f, on2 ? kmc[c] : 0.f);
+                lm2[c] = make_float2(PairArith<KT, PSI, true>::mask_term(on1 ? 1.f : 0.f),
+                                     PairArith<KT, PSI, true>::mask_term(on2 ? 1.f : 0.f));
+            }
+        } else {
+#pragma unroll
+            for (int c = 0; c < KT; ++c) {
+                km2[c] = f2(kmc[c]);
+                lm2[c] = f2(PairArith<KT, PSI, true>::mask_term(mkc[c]));
+            }
+        }
+
+        // phase 1: recompute
+        float2 z[L];
+        {
+            float2 vd[KT];
+#pragma unroll
+            for (int c = 0; c < KT; ++c) vd[c] = f2(0.f);
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) {
+                float xa[KT], xb[KT];
+                V::unpack(xring[tt * NT], xa);
+                V::unpack(xring[(L + tt) * NT], xb);
+                float2 y[KT];
+#pragma unroll
+                for (int c = 0; c < KT; ++c) {
+                    vd[c] = ffma2(f2(a[c]), vd[c], make_float2(xa[c], xb[c]));
+                    const float2 u = ffma2(vd[c], f2(iz[c]), f2(nxi[c]));
+                    if constexpr (PSI == PSI_MEXHAT) {
+                        const float2 ss = fmul2(u, u);
+                        const float2 t = fmul2(f2(kNegHalfLog2e), ss);
+                        const float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
+                        y[c] = ffma2(neg2(ss), e, e);
+                    } else {
+                        y[c] = make_float2(fabsf(u.x), fabsf(u.y));
+                    }
+                    hist[(tt * KT + c) * NT] = vd[c];
+                }
+                // the paired engine's tree: compartments (0, 2) and (1, 3), then the halves
+                float2 p = fmul2(km2[0], y[0]);
+                p = ffma2(km2[2], y[2], p);
+                float2 r = fmul2(km2[1], y[1]);
+                r = ffma2(km2[3], y[3], r);
+                float2 gv = fadd2(p, r);
+                gv.x = __fadd_rn(gv.x, __shfl_xor_sync(0xffffffffu, gv.x, 1));
+                gv.y = __fadd_rn(gv.y, __shfl_xor_sync(0xffffffffu, gv.y, 1));
+                z[tt] = gv;
+            }
+        }
+        fetch_x(q + 1, __fadd_rn(z[L - 1].x, z[L - 1].y));
+
+        // phase 2: the somas forward, then dL/dV^s backwards in time (dL/dZ = dL/dV^s)
+        float2 dz[L];
+        {
+            float v1 = 0.f, v2 = 0.f;
+            bool s1 = false, s2 = false;
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) {
+                v1 = soma_charge(z[tt].x, v1, s1, P);
+                v2 = soma_charge(z[tt].y, v2, s2, P);
+                s1 = v1 >= P.theta;
+                s2 = v2 >= P.theta;
+                z[tt] = make_float2(v1, v2);      // z now holds V^s
+            }
+            const float pi2 = 9.869604401089358f;
+            float2 dvn = f2(0.f);
+#pragma unroll
+            for (int tt = L - 1; tt >= 0; --tt) {
+                const float2 vs = z[tt];
+                const bool st1 = vs.x >= P.theta, st2 = vs.y >= P.theta;
+                if constexpr (BETA) {
+                    const float l1 = st1 ? (P.soft ? __fsub_rn(vs.x, P.theta) : 0.f) : vs.x;
+                    const float l2 = st2 ? (P.soft ? __fsub_rn(vs.y, P.theta) : 0.f) : vs.y;
+                    gb = ffma2(dvn, make_float2(l1, l2), gb);
+                }
+                const float2 dvds = ffma2(f2(kv), vs, f2(cs));
+                const float2 dvdv = make_float2(st1 ? b_spike : P.beta, st2 ? b_spike : P.beta);
+                const float2 ds = ffma2(dvds, dvn, make_float2(gring[tt * NT], gring[(L + tt) * NT]));
+                const float2 xd = make_float2(__fsub_rn(vs.x, P.theta), __fsub_rn(vs.y, P.theta));
+                const float2 qd = ffma2(fmul2(f2(pi2), xd), xd, f2(1.f));
+                const float2 sg = make_float2(fast_rcp(qd.x), fast_rcp(qd.y));
+                float2 dv = ffma2(sg, ds, fmul2(dvdv, dvn));
+                if (has_gv) {
+                    const float *gp = A.gv + j0 + (int64_t)k * jstep + (int64_t)tt * BN;
+                    dv = make_float2(__fadd_rn(dv.x, __ldcs(gp)), __fadd_rn(dv.y, two ? __ldcs(gp + jstep) : 0.f));
+                }
+                dz[tt] = dv;
+                dvn = dv;
+            }
+        }
+        fetch_gs(q + 1, __fadd_rn(dz[0].x, dz[0].y));
+
+        // phase 3: the dendritic reverse scan, one compartment at a time
+#pragma unroll
+        for (int c = 0; c < KT; ++c) {
+            float2 Ad = f2(0.f);
+            float2 vdt = hist[((L - 1) * KT + c) * NT];
+#pragma unroll
+            for (int tt = L - 1; tt >= 0; --tt) {
+                const float2 vdp = tt > 0 ? hist[((tt > 0 ? tt - 1 : 0) * KT + c) * NT] : f2(0.f);
+                const float2 u = ffma2(vdt, f2(iz[c]), f2(nxi[c]));
+                const float2 gy = fmul2(km2[c], dz[tt]);
+                float2 y, du;
+                if constexpr (PSI == PSI_MEXHAT) {
+                    const float2 ss = fmul2(u, u);
+                    const float2 t = ffma2(f2(kNegHalfLog2e), ss, lm2[c]);
+                    const float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
+                    y = ffma2(neg2(ss), e, e);
+                    const float2 w = fmul2(fadd2(ss, f2(-3.f)), e);
+                    du = fmul2(fmul2(w, u), gy);
+                } else {
+                    y = fmul2(lm2[c], make_float2(fabsf(u.x), fabsf(u.y)));
+                    du = make_float2(u.x > 0.f ? gy.x : (u.x < 0.f ? -gy.x : 0.f),
+                                     u.y > 0.f ? gy.y : (u.y < 0.f ? -gy.y : 0.f));
+                }
+                ngxi[c] = fadd2(ngxi[c], du);
+                ngz[c] = ffma2(u, du, ngz[c]);
+                gk[c] = ffma2(y, dz[tt], gk[c]);
+                Ad = ffma2(f2(a[c]), Ad, du);
+                ga[c] = ffma2(Ad, vdp, ga[c]);
+                hist[(tt * KT + c) * NT] = ffma2(Ad, f2(iz[c]), f2(0.f));
+                vdt = vdp;
+            }
+        }
+
+        // phase 4: dL/dX of each step and row as one vector
+        if (pos.active) {
+            float *g1 = gx0 + (int64_t)k * rX;
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) {
+                float ra[KT], rb[KT];
+#pragma unroll
+                for (int c = 0; c < KT; ++c) {
+                    const float2 h = hist[(tt * KT + c) * NT];
+                    ra[c] = h.x;
+                    rb[c] = h.y;
+                }
+                V::store(g1 + (int64_t)tt * sX, ks, ra);
+                if (two) V::store(g1 + rX + (int64_t)tt * sX, ks, rb);
+            }
+        }
+    }
+
+    // [alpha KT | xi KT | zeta KTb | kappa KTb | beta]; the first three carry 1/zeta here
+    constexpr int NA1 = NA + 1;
+    float v[NA1];
+#pragma unroll
+    for (int c = 0; c < KT; ++c) {
+        v[c] = __fmul_rn(__fadd_rn(ga[c].x, ga[c].y), iz[c]);
+        v[KT + c] = -__fmul_rn(__fadd_rn(ngxi[c].x, ngxi[c].y), iz[c]);
+        v[2 * KT + c] = -__fmul_rn(__fadd_rn(ngz[c].x, ngz[c].y), iz[c]);
+        v[3 * KT + c] = __fadd_rn(gk[c].x, gk[c].y);
+    }
+    v[NA] = (BETA && pos.sub == 0) ? __fadd_rn(gb.x, gb.y) : 0.f;
+#pragma unroll
+    for (int i = 0; i < NA1; ++i)
+        if (!pos.active || (i < KT && P.stateless)) v[i] = 0.f;
+    cp_async_wait<0>();
+    block_partials<KT, 1, LPN, NT>(g, pos, v, reinterpret_cast<float *>(sregion), A.partials);
+}
+
 // ---------------------------------------------------------------- launchers
 // Dynamic shared memory above 48 KB needs an explicit opt-in per kernel.
 template <typename Kern>
@@ -1768,6 +2049,17 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
         return cudaGetLastError();
     };
     auto go = [&](auto kernel) { return go_smem(kernel, smem); };
+    // 4-step rows of 8-compartment float32 neurons on two lanes: two rows per thread
+    constexpr bool kRowPair = DENDSN_BWD_ROWPAIR && K == 8 && G == 1 && XT == 0 && L == 4 && KT == 4;
+    if constexpr (kRowPair) {
+        if (a.g.T == 4 && !a.p.residual) {
+            const size_t rp = sizeof(float2) * L * KT * NT + xraw * 2 * L * NT +
+                              sizeof(float) * 2 * L * NT + sizeof(uint32_t) * 2 * NT;
+            const size_t rsm = red > rp ? red : rp;
+            return a.want_beta ? go_smem(dendsn_backward_rowpair_kernel<PSI, LAYOUT, true>, rsm)
+                               : go_smem(dendsn_backward_rowpair_kernel<PSI, LAYOUT, false>, rsm);
+        }
+    }
     // rows of one full chunk, a whole 8-compartment neuron per lane: the phased kernel
     // (deeper conv layer 738 -> 556 us; for the 4-compartment conv layer and for the token
     // layer on one 8-compartment lane it measured slower: 217 -> 280 us, 261 -> 295 us)

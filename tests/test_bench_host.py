@@ -40,7 +40,9 @@ def test_committed_traffic_record_names_kernels_the_layers_launch():
 def test_kernel_names_follow_the_library_plan():
     W = workloads.WORKLOADS
     assert bench.kernel_names(W["conv"]) == ("dendsn_forward_kernel", "dendsn_backward_kernel")
-    assert bench.kernel_names(W["token_dbg"]) == ("dendsn_forward_kernel", "dendsn_backward_kernel")
+    # 4-step rows of 8 float32 compartments on two lanes: two rows per thread
+    assert bench.kernel_names(W["token_dbg"]) == ("dendsn_forward_kernel", "dendsn_backward_rowpair_kernel")
+    assert bench.kernel_names(W["token_dbg"].with_(T=5))[1] == "dendsn_backward_kernel"
     assert bench.kernel_names(W["event"]) == ("dendsn_forward_kernel", "dendsn_backward_kernel")
     # rows of one full 8-step chunk, 8 bf16 compartments on one lane
     assert bench.kernel_names(W["deepconv_bf16"])[1] == "dendsn_backward_phased_kernel"

@@ -111,15 +111,19 @@ def test_variants(kw):
     check_layer(w)
 
 
+@pytest.mark.parametrize("T", [4, 8])
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("kw", [
-    dict(), dict(mask_p=0.5, mask_per_neuron=True), dict(reset="soft", psi="identity"),
-    dict(detach_reset=True), dict(stateless=True), dict(residual=True), dict(T=4),
+    dict(), dict(mask_p=0.5, mask_per_neuron=True), dict(mask_p=0.5),
+    dict(reset="soft", psi="identity"), dict(detach_reset=True), dict(stateless=True),
+    dict(residual=True), dict(layout="paper"),
 ], ids=lambda kw: "-".join(f"{k}={v}" for k, v in kw.items()) or "plain")
-def test_one_chunk_rows_of_whole_neurons(kw, dtype):
-    # T == 8 (or 4): rows of one full chunk, 8 compartments per lane -- the phased backward
-    # (the residual variant takes the chunked kernel)
-    w = workloads.Workload("phased", T=8, B=5, N=3 * 128, K=8, G=1, C=3, inner=128,
+def test_one_chunk_rows_of_8_compartments(kw, dtype, T):
+    # rows of one full chunk of 8-compartment neurons: the phased backward (bf16, or T == 8),
+    # and for float32 T == 4 the two-rows-per-thread backward of split lanes; B = 5 gives
+    # threads odd row counts (the unpaired last row); the residual variant takes the
+    # chunked kernel
+    w = workloads.Workload("onechunk", T=T, B=5, N=3 * 128, K=8, G=1, C=3, inner=128,
                            dtype=dtype, psi="mh", reset="hard", seed=41).with_(**kw)
     check_layer(w)
 
