@@ -6,9 +6,16 @@ x read, spikes written, grad_x and the four parameter gradients produced); with 
 ranks (torchrun) every rank processes its own batch and the parameter gradients
 are summed with one all-reduce (weak scaling).
 
+The headline is the long-horizon event-stream layer (T=64, B=32, 128 x 32 x 32
+neurons, K=4, float32, 80% zero inputs), the largest of the layer workloads. The
+same JSON line carries one block per other large layer workload (the conv layer,
+the deeper bf16 conv layer and the transformer-token layer with branch gating),
+each timed, roofline-checked and CPU-baselined the same way.
+
 Prints ONE JSON line on rank 0. Everything else goes to stderr.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload conv] [--impl ours|reference]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload event]
+                  [--blocks conv,deepconv_bf16,token_dbg] [--impl ours|reference]
 """
 from __future__ import annotations
 
@@ -33,6 +40,8 @@ FALLBACK_HBM_GBS = 6800.0
 L2_BYTES = 129 * 2**20
 FP32_LANES_PER_SM = 128          # float32 FMA lanes per Blackwell SM
 NOMINAL_SM_MHZ = 2070.0
+HEADLINE = "event"
+BLOCKS = ("conv", "deepconv_bf16", "token_dbg")
 
 
 def log(*a):
@@ -51,14 +60,18 @@ def parse_args():
                     help="learnable somatic decay: time dendsn_backward_plif (adds dL/dbeta)")
     ap.add_argument("--no-lif", action="store_true",
                     help="skip timing the point-neuron LIF layer baseline")
-    ap.add_argument("--workload", default="conv")
+    ap.add_argument("--workload", default=HEADLINE)
+    ap.add_argument("--blocks", default=None,
+                    help="comma-separated layer workloads timed after the headline and reported "
+                         "as blocks of the same line (default: the other large layers when the "
+                         "headline is the default one, else none; 'none' for none)")
     ap.add_argument("--psi", choices=["mh", "identity"], default=None)
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch B (smaller profiling captures)")
     ap.add_argument("--variant", choices=["stateful", "stateless", "resstateless", "resstateful"],
                     default="stateful", help="dendrite variant (Methods, DendSN variants)")
-    ap.add_argument("--cpu-seconds", type=float, default=12.0,
-                    help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--cpu-seconds", type=float, default=8.0,
+                    help="target CPU time of the oracle baseline sample of each layer")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -195,11 +208,55 @@ def recorded_traffic(kernel: str, workload: str):
 
 
 # ------------------------------------------------------------------ oracle (CPU baseline)
-def oracle_sample_rate(w, inp_cpu_fn, target_s: float):
-    """Times the float64 oracle (forward + backward) on a bounded sample of neurons.
+def host_cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the platform string)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            k, _, v = line.partition(":")
+            if k.strip() == "Model name" and v.strip():
+                vendor = next((l.partition(":")[2].strip() for l in out.splitlines()
+                               if l.partition(":")[0].strip() == "Vendor ID"), "")
+                return f"{vendor} {v.strip()}".strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                k, _, v = line.partition(":")
+                if k.strip().lower() in ("model name", "cpu model") and v.strip():
+                    return v.strip()
+    except OSError:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
 
-    Returns (neuron-steps/s, description of the sample, neuron-steps timed)."""
-    import numpy as np
+
+class pinned_to_one_core:
+    """Runs the enclosed block with this process restricted to one host core (the last one
+    it may use), then restores its affinity. Yields the core (None where affinity is not
+    available)."""
+
+    def __enter__(self):
+        self.saved = None
+        self.core = None
+        if hasattr(os, "sched_getaffinity"):
+            self.saved = os.sched_getaffinity(0)
+            self.core = max(self.saved)
+            os.sched_setaffinity(0, {self.core})
+        return self.core
+
+    def __exit__(self, *exc):
+        if self.saved is not None:
+            os.sched_setaffinity(0, self.saved)
+        return False
+
+
+def oracle_sample_rate(w, inp_cpu_fn, target_s: float):
+    """Times the float64 oracle (forward + backward) on a bounded sample of neurons, on one
+    host core.
+
+    Returns (neuron-steps/s, description of the sample, neuron-steps timed, seconds, core)."""
     import oracle
     oracle.build()
     ocfg = oracle.OracleConfig(T=w.T, K=w.K, G=w.G, C=w.C, psi=w.psi, reset=w.reset,
@@ -213,15 +270,17 @@ def oracle_sample_rate(w, inp_cpu_fn, target_s: float):
         oracle.backward(ocfg, x, chan, mrow, *prm, mask, gs)
         return time.perf_counter() - t
 
-    M = 256
-    dt = run(M)
-    while dt < 0.5 and M < w.B * w.N:
-        M = min(M * 4, w.B * w.N)
+    with pinned_to_one_core() as core:
+        M = 256
         dt = run(M)
-    M = int(min(w.B * w.N, max(1, M * target_s / max(dt, 1e-6))))
-    dt = run(M)
+        while dt < 0.3 and M < w.B * w.N:
+            M = min(M * 4, w.B * w.N)
+            dt = run(M)
+        M = int(min(w.B * w.N, max(1, M * target_s / max(dt, 1e-6))))
+        dt = run(M)
     ns = M * w.T
-    return ns / dt, f"{M} neurons x T={w.T} of the workload (forward + backward), 1 thread", ns, dt
+    return (ns / dt, f"{M} neurons x T={w.T} of the {w.name} layer (forward + backward), "
+            f"1 thread", ns, dt, core)
 
 
 def cpu_inputs_from(w, inp):
@@ -248,10 +307,17 @@ def cpu_inputs_from(w, inp):
     return fn
 
 
+def cpu_baseline_block(w, inp, target_s):
+    rate, sample, _, dt, core = oracle_sample_rate(w, cpu_inputs_from(w, inp), target_s)
+    return {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": sample + f", {dt:.1f} s", "pinned_core": core,
+            "cpu_model": host_cpu_model(), "host_cpus": os.cpu_count()}
+
+
 # ------------------------------------------------------------------ arms
-def workload_of(args):
+def workload_of(args, name=None):
     from paper_2412_06355_gb300.workloads import WORKLOADS
-    w = WORKLOADS[args.workload]
+    w = WORKLOADS[name or args.workload]
     if args.psi:
         w = w.with_(psi=args.psi)
     if args.batch:
@@ -262,9 +328,19 @@ def workload_of(args):
     return w
 
 
+def block_names(args):
+    """The layer workloads reported as blocks beside the headline."""
+    if args.blocks is None:
+        return list(BLOCKS) if args.workload == HEADLINE and not args.batch else []
+    if args.blocks.strip().lower() in ("", "none"):
+        return []
+    return [b.strip() for b in args.blocks.split(",") if b.strip() and b.strip() != args.workload]
+
+
 def config_dict(w, extra=None):
     d = {"workload": w.name, "T": w.T, "B": w.B, "N": w.N, "K": w.K, "G": w.G, "C": w.C,
-         "inner": w.inner, "x_dtype": w.dtype, "psi": w.psi, "reset": w.reset,
+         "inner": w.inner, "x_dtype": w.dtype, "state_dtype": "f32", "psi": w.psi,
+         "reset": w.reset,
          "mask": (None if w.mask_p is None else
                   f"Bernoulli({w.mask_p}) per {'neuron' if w.mask_per_neuron else 'channel'}"),
          "x_density": w.x_density, "layout": w.layout,
@@ -272,6 +348,12 @@ def config_dict(w, extra=None):
     if extra:
         d.update(extra)
     return d
+
+
+def dtype_label(w) -> str:
+    """The arithmetic type of the path: state and arithmetic are float32 for every layer;
+    the tensors in HBM are float32 or bfloat16."""
+    return "f32" if w.dtype == "f32" else "f32 (bf16 inputs/outputs, f32 state)"
 
 
 def slice_workload(w, M):
@@ -301,19 +383,20 @@ def run_reference(args):
 
     # size one step to about 90 s / (steps + warmup), between 0.2 s and 2 s
     per_step = max(0.2, min(2.0, 90.0 / max(args.steps + args.warmup, 1)))
-    probe = slice_workload(w, 4096)
-    pin = workloads.make_inputs(probe, "cpu")
-    t = time.perf_counter()
-    one_step(probe, pin)
-    rate = probe.neuron_steps / max(time.perf_counter() - t, 1e-6)
-    ws = slice_workload(w, int(rate * per_step / w.T))
-    inp = workloads.make_inputs(ws, "cpu")
-    for _ in range(args.warmup):
-        one_step(ws, inp)
-    t = time.perf_counter()
-    for _ in range(args.steps):
-        one_step(ws, inp)
-    dt = time.perf_counter() - t
+    with pinned_to_one_core() as core:
+        probe = slice_workload(w, 4096)
+        pin = workloads.make_inputs(probe, "cpu")
+        t = time.perf_counter()
+        one_step(probe, pin)
+        rate = probe.neuron_steps / max(time.perf_counter() - t, 1e-6)
+        ws = slice_workload(w, int(rate * per_step / w.T))
+        inp = workloads.make_inputs(ws, "cpu")
+        for _ in range(args.warmup):
+            one_step(ws, inp)
+        t = time.perf_counter()
+        for _ in range(args.steps):
+            one_step(ws, inp)
+        dt = time.perf_counter() - t
     value = args.steps * ws.neuron_steps / dt
     sample = (f"{ws.B * ws.N} neurons x T={w.T} per step ({ws.C} channels x {ws.inner}; a "
               f"slice of the {w.name} layer), float64 forward + backward, 1 thread")
@@ -324,7 +407,8 @@ def run_reference(args):
             "impl": "reference",
             "config": config_dict(w, {"sample_neurons_per_step": ws.B * ws.N}),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                             "sample": sample},
+                             "sample": sample, "pinned_core": core,
+                             "cpu_model": host_cpu_model(), "host_cpus": os.cpu_count()},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -367,85 +451,94 @@ def time_lif(T, B, N, dtype, steps, warmup, stream):
             "algorithmic_bytes_per_step": nbytes, "gbs": nbytes / (ms / 1e3) / 1e9}
 
 
-def run_ours(args):
-    import torch
-    import torch.distributed as dist
-    from paper_2412_06355_gb300 import binding, distributed, workloads
+class Layer:
+    """One layer workload resident on the device: inputs, outputs, workspaces and the
+    forward / backward calls of one step through the C ABI."""
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    if world > 1:
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl")
-    else:
-        torch.cuda.set_device(0)
-    dev = torch.device("cuda", torch.cuda.current_device())
-    w = workload_of(args)
-    w_rank = w.with_(seed=w.seed + 1000 * rank)
-    binding.load()
-    cfg = binding.config_of(w)
-    inp = workloads.make_inputs(w_rank, str(dev))
-    x, gs = inp["x"], inp["gs"]
-    alpha, xi, zeta, kappa, mask = (inp[k] for k in ("alpha", "xi", "zeta", "kappa", "mask"))
-    saved, scratch = binding.workspace(cfg, dev)
-    spikes = torch.empty((w.T, w.B, w.N), dtype=x.dtype, device=dev)
-    gx = torch.empty_like(x)
-    grads, views = distributed.param_grad_buffer(w.C, w.K, w.Kb, dev)
-    ga, gxi, gz, gk = (views[k] for k in ("galpha", "gxi", "gzeta", "gkappa"))
-    gbeta = torch.empty(w.C, dtype=torch.float32, device=dev)     # --plif: dL/dbeta
-    stream = torch.cuda.current_stream()
+    def __init__(self, w, args, dev, rank, stream):
+        import torch
+        from paper_2412_06355_gb300 import binding, distributed, workloads
+        self.w, self.args, self.stream = w, args, stream
+        self.w_rank = w.with_(seed=w.seed + 1000 * rank)
+        self.cfg = binding.config_of(w)
+        self.inp = workloads.make_inputs(self.w_rank, str(dev))
+        inp = self.inp
+        self.x, self.gs = inp["x"], inp["gs"]
+        self.prm = [inp[k] for k in ("alpha", "xi", "zeta", "kappa")]
+        self.mask = inp["mask"]
+        self.saved, self.scratch = binding.workspace(self.cfg, dev)
+        self.spikes = torch.empty((w.T, w.B, w.N), dtype=self.x.dtype, device=dev)
+        self.gx = torch.empty_like(self.x)
+        self.grads, views = distributed.param_grad_buffer(w.C, w.K, w.Kb, dev,
+                                                          with_beta=args.plif)
+        self.gviews = [views[k] for k in ("galpha", "gxi", "gzeta", "gkappa")]
+        self.gbeta = views.get("gbeta")
+        self.graphs = None
+        self.launches_per_step = None
 
-    def fwd(strm):
-        binding.dendsn_forward(cfg, x, alpha, xi, zeta, kappa, mask, spikes, None, saved, strm)
+    def fwd(self, strm):
+        from paper_2412_06355_gb300 import binding
+        if self.graphs is not None:
+            return self.graphs[0].replay()
+        binding.dendsn_forward(self.cfg, self.x, *self.prm, self.mask, self.spikes, None,
+                               self.saved, strm)
 
-    def bwd(strm):
-        if args.plif:
-            binding.dendsn_backward_plif(cfg, x, alpha, xi, zeta, kappa, mask, gs, None, saved,
-                                         gx, ga, gxi, gz, gk, gbeta, scratch, strm)
+    def bwd(self, strm):
+        from paper_2412_06355_gb300 import binding
+        if self.graphs is not None:
+            return self.graphs[1].replay()
+        if self.args.plif:
+            binding.dendsn_backward_plif(self.cfg, self.x, *self.prm, self.mask, self.gs, None,
+                                         self.saved, self.gx, *self.gviews, self.gbeta,
+                                         self.scratch, strm)
         else:
-            binding.dendsn_backward(cfg, x, alpha, xi, zeta, kappa, mask, gs, None, saved, gx,
-                                    ga, gxi, gz, gk, scratch, strm)
+            binding.dendsn_backward(self.cfg, self.x, *self.prm, self.mask, self.gs, None,
+                                    self.saved, self.gx, *self.gviews, self.scratch, strm)
 
-    # --graph: the forward and the backward each captured into a CUDA graph once, then
-    # replayed every step (no per-step host launch work; events stay between the replays)
-    launches_per_step = None
-    if args.graph:
-        if world > 1:
-            raise SystemExit("--graph times one GPU")
+    def capture(self):
+        """--graph: the forward and the backward each captured into a CUDA graph once, then
+        replayed every step (no per-step host launch work)."""
+        import torch
+        from paper_2412_06355_gb300 import binding
         side = torch.cuda.Stream()
-        side.wait_stream(stream)
+        side.wait_stream(self.stream)
         with torch.cuda.stream(side):               # one eager step before capturing
-            fwd(side)
-            bwd(side)
-        stream.wait_stream(side)
+            self.fwd(side)
+            self.bwd(side)
+        self.stream.wait_stream(side)
         torch.cuda.synchronize()
         n0 = binding.launch_count()
         graphs = []
-        for part in (fwd, bwd):
+        for part in (self.fwd, self.bwd):
             gr = torch.cuda.CUDAGraph()
             with torch.cuda.graph(gr):
                 part(torch.cuda.current_stream())
             graphs.append(gr)
-        launches_per_step = binding.launch_count() - n0
-        fwd = lambda strm: graphs[0].replay()     # noqa: E731  (replays on the current stream)
-        bwd = lambda strm: graphs[1].replay()     # noqa: E731
+        self.launches_per_step = binding.launch_count() - n0
+        self.graphs = graphs
+
+
+def time_layer(layer, args, world, dev):
+    """Warm-up, then exactly args.steps timed steps between barriers and synchronizes.
+    Returns the per-step event times, the whole-region time (max over ranks), the wall-clock
+    window and the launch count."""
+    import torch
+    import torch.distributed as dist
+    from paper_2412_06355_gb300 import binding, distributed
+    stream = layer.stream
 
     def step(ev=None):
         if ev is not None:
             ev[0].record(stream)
-        fwd(stream)
+        layer.fwd(stream)
         if ev is not None:
             ev[1].record(stream)
-        bwd(stream)
+        layer.bwd(stream)
         if ev is not None:
             ev[2].record(stream)
         if world > 1:
-            distributed.sum_param_grads(grads)
+            distributed.sum_param_grads(layer.grads)
 
-    clocks = ClockSampler(dev.index)
-    if rank == 0:
-        clocks.start()
     for _ in range(args.warmup):
         step()
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
@@ -462,116 +555,135 @@ def run_ours(args):
     torch.cuda.synchronize()
     t1 = time.time()
     n_launch = binding.launch_count() - n_launch0
-    if launches_per_step is not None:               # replays launch without library calls
-        n_launch = launches_per_step * args.steps
+    if layer.launches_per_step is not None:         # replays launch without library calls
+        n_launch = layer.launches_per_step * args.steps
     if world > 1:
         dist.barrier()
     ms = start.elapsed_time(end)
-    fwd_ms = [e[0].elapsed_time(e[1]) for e in ev]
-    bwd_ms = [e[1].elapsed_time(e[2]) for e in ev]
     if world > 1:
         t = torch.tensor([ms], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
-    clock = ClockSampler.summarize(clocks.stop(), t0, t1) if rank == 0 else None
+    return dict(ms=ms, fwd_ms=[e[0].elapsed_time(e[1]) for e in ev],
+                bwd_ms=[e[1].elapsed_time(e[2]) for e in ev], t0=t0, t1=t1, launches=n_launch)
 
-    # ---- end to end through the public API, host buffers, copies inside the timed region.
-    # The batch is held on the host as `nch` contiguous sub-batches (samples are independent);
-    # each sub-batch's H2D copy, forward + backward (C ABI, own stream) and D2H copy run on
-    # three streams ordered by events, so both copy directions overlap each other and the
-    # kernels. Parameter gradients come back per sub-batch and are summed on the host.
-    e2e = None
-    if not args.no_e2e:
-        nch = next(c for c in (8, 4, 2, 1) if w.B % c == 0)
-        bc = w.B // nch
-        wc = w_rank.with_(B=bc)
-        cfg_c = binding.config_of(wc)
-        pin = dict(pin_memory=True)
-        x_h = [torch.empty((w.T, bc) + tuple(x.shape[2:]), dtype=x.dtype, **pin) for _ in range(nch)]
-        gs_h = [torch.empty((w.T, bc, w.N), dtype=gs.dtype, **pin) for _ in range(nch)]
+
+def time_e2e(layer, args, world, dev):
+    """End to end through the C ABI from pinned host buffers, copies inside the timed region.
+
+    The batch is held on the host as `nch` contiguous sub-batches (samples are independent);
+    each sub-batch's H2D copy, forward + backward (C ABI, own stream) and D2H copy run on
+    three streams ordered by events, so both copy directions overlap each other and the
+    kernels. Every sub-batch call has the whole layer's columns, B / nch samples. Each
+    step's parameter gradients come back per sub-batch and are summed on the host while the
+    next step runs; the last step's sum is done before the clock stops. Timed on the wall
+    clock (host work included)."""
+    import torch
+    import torch.distributed as dist
+    from paper_2412_06355_gb300 import binding, distributed
+    w, x, gs = layer.w, layer.x, layer.gs
+    alpha, xi, zeta, kappa = layer.prm
+    mask = layer.mask
+    nch = next(c for c in (8, 4, 2, 1) if w.B % c == 0)
+    bc = w.B // nch
+    wc = layer.w_rank.with_(B=bc)
+    cfg_c = binding.config_of(wc)
+    pin = dict(pin_memory=True)
+    x_h = [torch.empty((w.T, bc) + tuple(x.shape[2:]), dtype=x.dtype, **pin) for _ in range(nch)]
+    gs_h = [torch.empty((w.T, bc, w.N), dtype=gs.dtype, **pin) for _ in range(nch)]
+    for c in range(nch):
+        x_h[c].copy_(x[:, c * bc:(c + 1) * bc])
+        gs_h[c].copy_(gs[:, c * bc:(c + 1) * bc])
+    x_d = [torch.empty_like(t, device=dev) for t in x_h]
+    gs_d = [torch.empty_like(t, device=dev) for t in gs_h]
+    s_d = [torch.empty((w.T, bc, w.N), dtype=x.dtype, device=dev) for _ in range(nch)]
+    gx_d = [torch.empty_like(t) for t in x_d]
+    ws_c = [binding.workspace(cfg_c, dev) for _ in range(nch)]
+    ng = layer.grads.numel()
+    g_d = torch.empty((nch, ng), dtype=torch.float32, device=dev)
+    g_v = [distributed.split_param_grads(g_d[c], w.C, w.K, w.Kb) for c in range(nch)]
+    s_h = [torch.empty(t.shape, dtype=t.dtype, **pin) for t in s_d]
+    gx_h = [torch.empty(t.shape, dtype=t.dtype, **pin) for t in gx_d]
+    g_h = [torch.empty((nch, ng), dtype=torch.float32, **pin) for _ in range(2)]
+    h2d = sum(t.numel() * t.element_size() for t in x_h + gs_h)
+    d2h = (sum(t.numel() * t.element_size() for t in s_h + gx_h) +
+           g_h[0].numel() * g_h[0].element_size())
+    up, comp, down = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    ev = lambda: torch.cuda.Event()                   # noqa: E731
+    loaded, computed, returned = ([ev() for _ in range(nch)] for _ in range(3))
+    all_done, grads_home = ev(), [ev(), ev()]
+    sums = []
+
+    def e2e_step(k):
         for c in range(nch):
-            x_h[c].copy_(x[:, c * bc:(c + 1) * bc])
-            gs_h[c].copy_(gs[:, c * bc:(c + 1) * bc])
-        x_d = [torch.empty_like(t, device=dev) for t in x_h]
-        gs_d = [torch.empty_like(t, device=dev) for t in gs_h]
-        s_d = [torch.empty((w.T, bc, w.N), dtype=x.dtype, device=dev) for _ in range(nch)]
-        gx_d = [torch.empty_like(t) for t in x_d]
-        ws_c = [binding.workspace(cfg_c, dev) for _ in range(nch)]
-        ng = grads.numel()
-        g_d = torch.empty((nch, ng), dtype=grads.dtype, device=dev)
-        g_v = [distributed.split_param_grads(g_d[c], w.C, w.K, w.Kb) for c in range(nch)]
-        s_h = [torch.empty(t.shape, dtype=t.dtype, **pin) for t in s_d]
-        gx_h = [torch.empty(t.shape, dtype=t.dtype, **pin) for t in gx_d]
-        g_h = torch.empty((nch, ng), dtype=grads.dtype, **pin)
-        h2d = sum(t.numel() * t.element_size() for t in x_h + gs_h)
-        d2h = (sum(t.numel() * t.element_size() for t in s_h + gx_h) +
-               g_h.numel() * g_h.element_size())
-        up, comp, down = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
-        ev = lambda: torch.cuda.Event()
-        loaded, computed, returned = ([ev() for _ in range(nch)] for _ in range(3))
-        all_done = ev()
-
-        def e2e_step():
-            for c in range(nch):
-                with torch.cuda.stream(up):
-                    up.wait_event(computed[c])           # the previous step has read x_d[c]
-                    x_d[c].copy_(x_h[c], non_blocking=True)
-                    gs_d[c].copy_(gs_h[c], non_blocking=True)
-                    loaded[c].record(up)
-                comp.wait_event(loaded[c])
-                comp.wait_event(returned[c])             # the previous step's D2H is done
-                saved_c, scratch_c = ws_c[c]
-                binding.dendsn_forward(cfg_c, x_d[c], alpha, xi, zeta, kappa, mask, s_d[c], None,
-                                       saved_c, comp)
-                binding.dendsn_backward(cfg_c, x_d[c], alpha, xi, zeta, kappa, mask, gs_d[c], None,
-                                        saved_c, gx_d[c], *g_v[c], scratch_c, comp)
-                computed[c].record(comp)
-                with torch.cuda.stream(down):
-                    down.wait_event(computed[c])
-                    s_h[c].copy_(s_d[c], non_blocking=True)
-                    gx_h[c].copy_(gx_d[c], non_blocking=True)
-                    returned[c].record(down)
-            if world > 1:
-                with torch.cuda.stream(comp):
-                    dist.all_reduce(g_d)                 # sums every sub-batch's row over ranks
-            all_done.record(comp)
+            with torch.cuda.stream(up):
+                up.wait_event(computed[c])           # the previous step has read x_d[c]
+                x_d[c].copy_(x_h[c], non_blocking=True)
+                gs_d[c].copy_(gs_h[c], non_blocking=True)
+                loaded[c].record(up)
+            comp.wait_event(loaded[c])
+            comp.wait_event(returned[c])             # the previous step's D2H is done
+            saved_c, scratch_c = ws_c[c]
+            binding.dendsn_forward(cfg_c, x_d[c], alpha, xi, zeta, kappa, mask, s_d[c], None,
+                                   saved_c, comp)
+            binding.dendsn_backward(cfg_c, x_d[c], alpha, xi, zeta, kappa, mask, gs_d[c], None,
+                                    saved_c, gx_d[c], *g_v[c], scratch_c, comp)
+            computed[c].record(comp)
             with torch.cuda.stream(down):
-                down.wait_event(all_done)
-                g_h.copy_(g_d, non_blocking=True)
-
-        ke = max(3, min(args.steps, 20))
-        for _ in range(3):
-            e2e_step()
+                down.wait_event(computed[c])
+                s_h[c].copy_(s_d[c], non_blocking=True)
+                gx_h[c].copy_(gx_d[c], non_blocking=True)
+                returned[c].record(down)
         if world > 1:
-            dist.barrier()
-        torch.cuda.synchronize()
-        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        s0.record(up)
-        for _ in range(ke):
-            e2e_step()
-        s1.record(down)
-        torch.cuda.synchronize()
-        ems = s0.elapsed_time(s1)
-        g_sum = g_h.sum(dim=0)                           # the step's parameter gradients
-        assert torch.isfinite(g_sum).all()
-        if world > 1:
-            t = torch.tensor([ems], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ems = float(t.item())
-        e2e = {"value": world * ke * w.neuron_steps / (ems / 1e3), "unit": UNIT,
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": ke,
-               "sub_batches": nch, "streams": 3}
+            with torch.cuda.stream(comp):
+                dist.all_reduce(g_d)                 # sums every sub-batch's row over ranks
+        all_done.record(comp)
+        with torch.cuda.stream(down):
+            down.wait_event(all_done)
+            g_h[k % 2].copy_(g_d, non_blocking=True)
+            grads_home[k % 2].record(down)
 
-    if rank != 0:
-        if world > 1:
-            dist.destroy_process_group()
-        return
+    def host_sum(k):                                 # the step's parameter gradients
+        grads_home[k % 2].synchronize()
+        sums.append(g_h[k % 2].sum(dim=0))
 
-    # ---- roofline of the dominant kernel
+    ke = max(3, min(args.steps, 20))
+    for k in range(3):
+        e2e_step(k)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    sums.clear()
+    t0 = time.perf_counter()
+    for k in range(ke):
+        e2e_step(k)
+        if k > 0:
+            host_sum(k - 1)
+    host_sum(ke - 1)
+    torch.cuda.synchronize()
+    ems = (time.perf_counter() - t0) * 1e3
+    assert len(sums) == ke and all(bool(torch.isfinite(s).all()) for s in sums)
+    if world > 1:
+        t = torch.tensor([ems], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ems = float(t.item())
+    return {"value": world * ke * w.neuron_steps / (ems / 1e3), "unit": UNIT,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": ke,
+            "ms_per_step": ems / ke, "sub_batches": nch, "sub_batch_B": bc, "streams": 3,
+            "timing": "wall clock; the per-sub-batch parameter gradients are summed on the "
+                      "host inside the timed region",
+            "launch_geometry": f"{nch} calls of B={bc} per step (the timed headline is one "
+                               f"call of B={w.B})"}
+
+
+def layer_report(layer, timing, world, dev, peak, peak_kind, clock):
+    """Roofline of the dominant kernel, the step's HBM fraction and the throughput of one
+    layer from its timing."""
+    import torch
+    w = layer.w
     ab = w.algorithmic_bytes()
     ops = w.fp32_ops_per_neuron_step()
-    fwd_avg, bwd_avg = statistics.mean(fwd_ms), statistics.mean(bwd_ms)
-    peak, peak_kind = measured_hbm_peak()
+    fwd_avg, bwd_avg = statistics.mean(timing["fwd_ms"]), statistics.mean(timing["bwd_ms"])
     fname, bname = kernel_names(w)
     if bwd_avg >= fwd_avg:
         kname, kbytes, kms, kops = bname, ab["backward"], bwd_avg, ops["backward"]
@@ -581,7 +693,8 @@ def run_ours(args):
     # the float32 roof of the same kernel: its float32 operations (a cost model counted from
     # the equations) against SMs x 128 FMA lanes x the SM clock
     sm_mhz = (clock or {}).get("sm_max_mhz") or NOMINAL_SM_MHZ
-    fp32_peak = torch.cuda.get_device_properties(dev).multi_processor_count * FP32_LANES_PER_SM * sm_mhz * 1e6
+    fp32_peak = (torch.cuda.get_device_properties(dev).multi_processor_count *
+                 FP32_LANES_PER_SM * sm_mhz * 1e6)
     ops_launch = kops * w.neuron_steps
     t_hbm, t_alu = kbytes / (peak * 1e9), ops_launch / fp32_peak
     alu = {"fp32_ops_per_neuron_step": kops, "fp32_ops_per_launch": ops_launch,
@@ -589,60 +702,134 @@ def run_ours(args):
            "frac": ops_launch / (kms / 1e3) / fp32_peak,
            "peak_basis": f"SMs x {FP32_LANES_PER_SM} FP32 lanes x {sm_mhz:.0f} MHz",
            "min_ms_at_fp32_peak": t_alu * 1e3, "min_ms_at_hbm_peak": t_hbm * 1e3}
-    step_ms = ms / args.steps
+    step_ms = timing["ms"] / layer.args.steps
     value = world * w.neuron_steps / (step_ms / 1e3)
-    cpu = None
-    if not args.no_cpu_baseline and world == 1:
-        rate, sample, _, dt = oracle_sample_rate(w, cpu_inputs_from(w, inp), args.cpu_seconds)
-        cpu = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
-               "sample": sample + f", {dt:.1f} s", "host_cpus": os.cpu_count()}
+    ab_unit = kbytes / w.neuron_steps
+    roof = {**({"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peak,
+                "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak}
+               if t_hbm >= t_alu else
+               {"bound": "alu", "kernel": kname, "achieved": alu["achieved_tops"],
+                "peak": alu["peak_tops"], "peak_kind": alu["peak_basis"],
+                "unit": "FP32 Top/s", "frac": alu["frac"]}),
+            "hbm_frac": achieved / peak,
+            "frac_of_8tbs": achieved / NOMINAL_HBM_GBS,
+            "alu": alu,
+            # counters were taken on the plain backward build, not the dL/dbeta one
+            "traffic": None if layer.args.plif else recorded_traffic(kname, w.name),
+            "algorithmic_bytes_per_neuron_step": ab_unit,
+            "neuron_steps_per_launch": w.neuron_steps,
+            "algorithmic_bytes_per_launch": kbytes, "avg_launch_ms": kms}
+    hbm = {"algorithmic_bytes_per_step": ab["total"],
+           "step_gbs": ab["total"] / (step_ms / 1e3) / 1e9,
+           "frac_of_8tbs": ab["total"] / (step_ms / 1e3) / 1e9 / NOMINAL_HBM_GBS,
+           "frac_of_measured": ab["total"] / (step_ms / 1e3) / 1e9 / peak,
+           "forward_ms": fwd_avg, "backward_ms": bwd_avg}
+    return value, step_ms, roof, hbm
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2412_06355_gb300 import binding
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    if args.graph and world > 1:
+        raise SystemExit("--graph times one GPU")
+    dev = torch.device("cuda", torch.cuda.current_device())
+    binding.load()
+    stream = torch.cuda.current_stream()
+    peak, peak_kind = measured_hbm_peak()
+    clocks = ClockSampler(dev.index)
+    if rank == 0:
+        clocks.start()
+
+    names = [args.workload] + block_names(args)
+    results = []                                     # (layer workload, timing, e2e)
+    e2e = None
+    for i, name in enumerate(names):
+        w = workload_of(args, name)
+        layer = Layer(w, args, dev, rank, stream)
+        if args.graph:
+            layer.capture()
+        timing = time_layer(layer, args, world, dev)
+        if i == 0 and not args.no_e2e:
+            e2e = time_e2e(layer, args, world, dev)
+        cpu = None
+        results.append([layer, timing, cpu])
+        log(f"{name}: {timing['ms'] / args.steps:.4f} ms per step")
+        if i > 0:
+            # the layer's device buffers go before the next one is drawn; the host-side CPU
+            # baseline sample is drawn from the inputs later, so keep only what it needs
+            layer.saved = layer.scratch = layer.spikes = layer.gx = None
+    clock_rows = clocks.stop() if rank == 0 else []
+
     lif = None
-    if not args.no_lif:
+    if rank == 0 and not args.no_lif:
         # the paper compares DendSN with LIF layers (Results, efficiency paragraph): here a
-        # LIF layer with the same neurons (one current each), and one fed the same input
-        # tensor (N*K point neurons)
+        # LIF layer with the same neurons as the conv layer (one current each), and one fed
+        # the same input tensor (N*K point neurons)
+        wl = next((r[0].w for r in results if r[0].w.name == "conv"), results[0][0].w)
+        lay = next(r for r in results if r[0].w is wl)
         steps_l = max(3, min(args.steps, 50))
-        same_n = time_lif(w.T, w.B, w.N, w.dtype, steps_l, 3, stream)
-        same_x = time_lif(w.T, w.B, w.N * w.K, w.dtype, steps_l, 3, stream)
+        same_n = time_lif(wl.T, wl.B, wl.N, wl.dtype, steps_l, 3, stream)
+        same_x = time_lif(wl.T, wl.B, wl.N * wl.K, wl.dtype, steps_l, 3, stream)
         for d in (same_n, same_x):
             d["frac_of_measured"] = d["gbs"] / peak
-        lif = {"same_neurons": same_n, "same_input": same_x,
-               "dendsn_over_lif_same_neurons": value / world / same_n["value"],
-               "dendsn_over_lif_same_input": same_x["ms_per_step"] / step_ms,
+        step_ms_l = lay[1]["ms"] / args.steps
+        lif = {"workload": wl.name, "same_neurons": same_n, "same_input": same_x,
+               "dendsn_over_lif_same_neurons": (wl.neuron_steps / (step_ms_l / 1e3)) /
+                                               same_n["value"],
+               "dendsn_over_lif_same_input": same_x["ms_per_step"] / step_ms_l,
                "note": "layer-level ratios of fwd+bwd throughput; the paper's 0.92 is for "
                        "whole networks (Tiny ImageNet VGG, Triton kernels)"}
-    x_bytes = x.numel() * x.element_size()
-    line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": config_dict(w, {
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    # CPU baselines last: the oracle runs pinned to one host core after all GPU timing
+    blocks = []
+    head = None
+    for i, (layer, timing, _) in enumerate(results):
+        w = layer.w
+        clock = ClockSampler.summarize(clock_rows, timing["t0"], timing["t1"])
+        value, step_ms, roof, hbm = layer_report(layer, timing, world, dev, peak, peak_kind,
+                                                 clock)
+        cpu = None
+        if not args.no_cpu_baseline and world == 1:
+            cpu = cpu_baseline_block(w, layer.inp, args.cpu_seconds)
+        x_bytes = layer.x.numel() * layer.x.element_size()
+        cfg = config_dict(w, {
             "l2": f"inputs larger than L2: x is {x_bytes / 2**20:.0f} MiB per step "
                   f"(L2 {L2_BYTES // 2**20} MiB), no flush",
             "parallelism": f"dp{world}" if world > 1 else "single GPU",
             "soma": "plif (learnable beta)" if args.plif else "lif",
-            "launch": "cuda graph replay" if args.graph else "eager"}),
-        "roofline": {**({"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peak,
-                         "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak}
-                        if t_hbm >= t_alu else
-                        {"bound": "alu", "kernel": kname, "achieved": alu["achieved_tops"],
-                         "peak": alu["peak_tops"], "peak_kind": alu["peak_basis"],
-                         "unit": "FP32 Top/s", "frac": alu["frac"]}),
-                     "hbm_frac": achieved / peak,
-                     "alu": alu,
-                     # counters were taken on the plain backward build, not the dL/dbeta one
-                     "traffic": None if args.plif else recorded_traffic(kname, w.name),
-                     "algorithmic_bytes_per_launch": kbytes, "avg_launch_ms": kms},
-        "hbm": {"algorithmic_bytes_per_step": ab["total"],
-                "step_gbs": ab["total"] / (step_ms / 1e3) / 1e9,
-                "frac_of_8tbs": ab["total"] / (step_ms / 1e3) / 1e9 / NOMINAL_HBM_GBS,
-                "frac_of_measured": ab["total"] / (step_ms / 1e3) / 1e9 / peak,
-                "forward_ms": fwd_avg, "backward_ms": bwd_avg},
-        "clocks": clock,
-        "e2e": e2e,
-        "gpu_launches": n_launch,
-        "cpu_baseline": cpu,
-        "lif_baseline": lif,
+            "launch": "cuda graph replay" if args.graph else "eager"})
+        block = {"workload": w.name, "value": value, "unit": UNIT, "ms_per_step": step_ms,
+                 "forward_ms": hbm["forward_ms"], "backward_ms": hbm["backward_ms"],
+                 "dtype": dtype_label(w), "config": cfg, "roofline": roof, "hbm": hbm,
+                 "clocks": clock, "gpu_launches": timing["launches"], "cpu_baseline": cpu}
+        if i == 0:
+            head = block
+        else:
+            blocks.append(block)
+
+    line = {
+        "metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": head["ms_per_step"],
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": head["dtype"], "data": "synthetic", "config": head["config"],
+        "roofline": head["roofline"], "hbm": head["hbm"], "clocks": head["clocks"],
+        "e2e": e2e, "gpu_launches": head["gpu_launches"], "cpu_baseline": head["cpu_baseline"],
+        "blocks": blocks, "lif_baseline": lif,
     }
     print(json.dumps(line), flush=True)
     if world > 1:

@@ -176,6 +176,10 @@ dendsn_status dendsn_backward_plif(const dendsn_config *cfg, const void *x, cons
  *     is rejected with DENDSN_ERR_UNSUPPORTED before anything is enqueued.
  *   - The first call on a device looks up that buffer's device address (with that
  *     device current) and caches it; make that first call before any stream capture.
+ *     The cached address belongs to the device's context at that time: after a
+ *     cudaDeviceReset on that device (which unloads the library's device code) it is
+ *     stale, so a process that resets a device must not call this entry point on it
+ *     again.
  *   - All calls share the one buffer, which keeps the last call's contents. Nothing in
  *     it needs to start at zero. Calls whose executions overlap on the GPU (for example
  *     on two streams without ordering between them) race on it and give wrong results.

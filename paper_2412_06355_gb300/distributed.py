@@ -2,8 +2,9 @@
 
 Neurons are independent, so a batch splits across ranks with no exchange in the
 forward; the only exchange is the sum of the parameter gradients (2K + 2Kb floats
-per channel) after the backward. These helpers hold that host-side logic; the
-arithmetic stays in the CUDA library.
+per channel, plus one for dL/dbeta when the somatic decay is learnable) after the
+backward. These helpers hold that host-side logic; the arithmetic stays in the CUDA
+library.
 """
 from __future__ import annotations
 
@@ -22,21 +23,32 @@ def shard_range(n: int, world: int, rank: int) -> Tuple[int, int]:
     return start, start + base + (1 if rank < extra else 0)
 
 
-def param_grad_buffer(C: int, K: int, Kb: int, device=None) -> Tuple[torch.Tensor, Dict[str, torch.Tensor]]:
-    """One flat float32 buffer holding the four parameter gradients, and views into it.
+def _sizes(C: int, K: int, Kb: int, with_beta: bool):
+    return [C * K, C * K, C * Kb, C * Kb] + ([C] if with_beta else [])
 
-    A single buffer lets one all-reduce sum all four.
+
+def param_grad_buffer(C: int, K: int, Kb: int, device=None, with_beta: bool = False
+                      ) -> Tuple[torch.Tensor, Dict[str, torch.Tensor]]:
+    """One flat float32 buffer holding the parameter gradients, and views into it.
+
+    galpha, gxi [C, K], gzeta, gkappa [C, Kb], and with_beta also gbeta [C] (the
+    per-channel dL/dbeta of a learnable somatic decay). A single buffer lets one
+    all-reduce sum all of them.
     """
-    flat = torch.zeros(2 * C * K + 2 * C * Kb, dtype=torch.float32, device=device)
-    ga, gxi, gz, gk = torch.split(flat, [C * K, C * K, C * Kb, C * Kb])
-    return flat, {"galpha": ga.view(C, K), "gxi": gxi.view(C, K), "gzeta": gz.view(C, Kb),
-                  "gkappa": gk.view(C, Kb)}
+    flat = torch.zeros(sum(_sizes(C, K, Kb, with_beta)), dtype=torch.float32, device=device)
+    return flat, split_param_grads(flat, C, K, Kb, with_beta, as_dict=True)
 
 
-def split_param_grads(flat: torch.Tensor, C: int, K: int, Kb: int):
-    """(galpha, gxi, gzeta, gkappa) views of one flat parameter-gradient row."""
-    ga, gxi, gz, gk = torch.split(flat, [C * K, C * K, C * Kb, C * Kb])
-    return ga.view(C, K), gxi.view(C, K), gz.view(C, Kb), gk.view(C, Kb)
+def split_param_grads(flat: torch.Tensor, C: int, K: int, Kb: int, with_beta: bool = False,
+                      as_dict: bool = False):
+    """Views of one flat parameter-gradient row: (galpha, gxi, gzeta, gkappa[, gbeta]), or a
+    dict with those keys."""
+    parts = torch.split(flat, _sizes(C, K, Kb, with_beta))
+    views = [parts[0].view(C, K), parts[1].view(C, K), parts[2].view(C, Kb),
+             parts[3].view(C, Kb)] + ([parts[4]] if with_beta else [])
+    if as_dict:
+        return dict(zip(("galpha", "gxi", "gzeta", "gkappa", "gbeta"), views))
+    return tuple(views)
 
 
 def sum_param_grads(flat: torch.Tensor, group=None) -> torch.Tensor:

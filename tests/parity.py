@@ -1,36 +1,40 @@
 """Shared machinery of the GPU-vs-oracle parity tests.
 
-Tolerances (written here once, used by every parity test):
-  V^s      |gpu - oracle| <= 1e-6 + 1e-5 |oracle| (+ the soma allowance below)
+Bounds (written here once, used by every parity test). By default a layer is checked at
+the stated bounds:
+  V^s      |gpu - oracle| <= 1e-6 + 1e-5 |oracle|
   spikes   identical, except at and after a step where the oracle's potential lies
            within 1e-5 of the threshold (an "ambiguous" step: float32 rounding may
            legitimately decide it either way)
-  grads    |gpu - oracle| <= rtol |oracle| + atol_rel * rms(oracle)
-           float32: rtol 1e-4, atol_rel 1e-5;  bfloat16 grad_x: rtol 2e-2, atol_rel 1e-2
-           parameter gradients (float32 sums over up to 10^6 terms): rtol 1e-4,
-           atol_rel 1e-5
-  atol_rel: an element that is a near-cancelling sum of terms of size ~rms carries
-  an absolute float32 rounding error ~(number of terms) * 6e-8 * rms, so a pure
-  relative bound is meaningless for it; 1e-5 * rms covers sums of up to ~150
-  terms. grad_x is the compartment scan (memory 1 / (1 - alpha)) of terms that are
-  themselves the soma's reverse scan (memory 1 / (1 - beta)), so its atol_rel is
-  max(1e-5, eps32 / ((1 - alpha_max)(1 - beta))): 1e-5 for beta = 0.5, 2.4e-5 for the
-  long-horizon layers with alpha, beta = 0.95 (~400 effective terms).
+  params   |gpu - oracle| <= 1e-4 |oracle| + 1e-6 rms(oracle tensor)
+  grad_x   |gpu - oracle| <= rtol |oracle| + 1e-5 rms(oracle tensor), rtol 1e-4 (float32)
+           or 2e-2 (bfloat16)
+The absolute term of grad_x is a reading, not the stated 1e-6 rms. An element of dL/dX is
+a sum, over later steps, of products of the soma's reverse recursion (Eq. methods-sg, memory
+1 / (1 - beta)) and the compartment scan (memory 1 / (1 - alpha), up to 20), tens of terms
+of size ~rms; float32 evaluation rounds each at a few units of 2^-24, and the spike
+surrogate's slope (up to 2.04) turns V^s's own float32 rounding into more, so an element
+whose terms nearly cancel carries an absolute error of a few 1e-6 rms. A plain float32
+restatement of the method (tests/f32_restatement.py: IEEE float32 operations, correctly
+rounded exponential) misses 1e-6 rms on all four large layer workloads, by up to 2.9x, and
+meets 1e-5 rms with a margin of at least 2.3x (tests/test_f32_restatement.py); 1e-5 is the
+smallest decade that float32 arithmetic meets. Parameter gradients meet the stated bound.
+
+Layers with a long horizon and a slow somatic decay (T >= 256 and beta >= 0.9: the L5PC-like
+layers and the time-parallel fuzz cases) are checked with three derived allowances instead
+(needs_allowance): there a plain float32 restatement itself misses the stated V^s bound
+(by up to 3.4x) or even the grad_x reading (by up to 2.4x, identity branches), as
+tests/test_f32_restatement.py shows. The allowances:
 
 V^s gets a per-element allowance on top of 1e-6 + 1e-5 |v|. The soma recursion
 V[t] = beta leak[t-1] + Z[t] (Eq. methods-lif-reset-charge) adds a float32 rounding of about
 eps32 (|Z[t]| + |V[t]|) per step and carries earlier ones with weight beta (cut by a hard
 reset), and Z[t] inherits the compartment scan's rounding (about eps32 sum_k alpha^k |X|)
-through kappa m |psi'| / zeta. With beta = 0.95 and a soft reset that reaches several 1e-6 where
-V^s itself is near zero, and a plain sequential float32 restatement misses the bare bound
-there too. The allowance is 2x that first-order error: a median 5e-7 on the beta = 0.5 conv
-layer (a tenth of the bare bound there). A step is ambiguous when the oracle's V^s lies within max(1e-5, that V^s tolerance)
-of theta.
-
-Neurons whose oracle trajectory has an ambiguous step get zero upstream gradient
-(grad_spikes and grad_v) on BOTH sides: the backward is linear in them, so those
-neurons then contribute exactly zero to every gradient whatever spike pattern
-each side followed, and the remaining comparisons stay exact-trajectory ones.
+through kappa m |psi'| / zeta. With beta = 0.95 and a soft reset that reaches several 1e-6
+where V^s itself is near zero. The allowance is 2x that first-order error. A step is
+ambiguous when the oracle's V^s lies within max(1e-5, that V^s tolerance) of theta.
+grad_x's atol_rel becomes max(1e-5, eps32 / ((1 - alpha_max)(1 - beta))) (the nested scans:
+~400 effective terms at alpha, beta = 0.95), the parameter gradients' 1e-5.
 
 grad_x with an identity branch nonlinearity gets one more, per-element allowance. The
 branch gradient there is dr_b * u_i / r_b (Eq. methods-branch-aggregation): as the
@@ -39,8 +43,12 @@ u_i = (V^d_i - xi_i) / zeta_b, about eps32 (|V^d_i| / (1 - alpha_i) + |xi_i|) / 
 (V^d's own accumulated rounding included), divided by r_b, and nothing damps it (the
 Mexican hat's psi'(r) ~ r does). The allowance is 4x that first-order error, times
 |kappa_b m_b dL/dV^s[t]| / zeta_b, carried back through the compartment scan like the
-gradient itself. It is negligible except within ~1e-3 of r_b = 0 (a plain float32
-restatement of the backward exceeds the bare bound there too).
+gradient itself. It is negligible except within ~1e-3 of r_b = 0.
+
+Neurons whose oracle trajectory has an ambiguous step get zero upstream gradient
+(grad_spikes and grad_v) on BOTH sides: the backward is linear in them, so those
+neurons then contribute exactly zero to every gradient whatever spike pattern
+each side followed, and the remaining comparisons stay exact-trajectory ones.
 """
 from __future__ import annotations
 
@@ -52,8 +60,12 @@ from paper_2412_06355_gb300 import binding, workloads
 
 AMBIGUOUS = 1e-5
 V_RTOL, V_ATOL = 1e-5, 1e-6
-G_RTOL, G_ATOL_REL = 1e-4, 1e-5
-BF16_RTOL, BF16_ATOL_REL = 2e-2, 1e-2
+G_RTOL = 1e-4
+GX_ATOL_REL = 1e-5        # grad_x (the reading above)
+P_ATOL_REL = 1e-6         # parameter gradients (stated)
+BF16_RTOL = 2e-2
+G_ATOL_REL = 1e-5         # the allowance mode's gradient atol_rel
+BF16_ATOL_REL = 1e-2      # the allowance mode's bfloat16 grad_x atol_rel
 
 
 def rms(a: np.ndarray) -> float:
@@ -202,17 +214,31 @@ def run_gpu(w, inp_dev: dict, gs, gv, want_v=True):
     return out
 
 
-def check_layer(w, seed_inputs=None, with_gv=True):
-    """Full parity check of workload `w` (all neurons) against the oracle."""
+def needs_allowance(w) -> bool:
+    """A long horizon at a slow somatic decay, where float32 evaluation itself misses the
+    stated bounds (see the module docstring)."""
+    return w.T >= 256 and w.beta >= 0.9
+
+
+def check_layer(w, seed_inputs=None, with_gv=True, allowance=None):
+    """Full parity check of workload `w` (all neurons) against the oracle, at the stated
+    bounds, or with the derived allowances when `allowance` (default: needs_allowance(w);
+    see the module docstring)."""
+    if allowance is None:
+        allowance = needs_allowance(w)
     inp = seed_inputs if seed_inputs is not None else workloads.make_inputs(w, "cpu", with_gv=with_gv)
     s_o, v_o = oracle.forward_layer(w, inp)
     chan, mrow = oracle.layer_channels(w.B, w.N, w.C, w.inner, w.mask_per_neuron)
     xk = oracle.layer_x(w, inp["x"])
-    v_extra = soma_rounding_allowance(w, xk, chan, mrow, inp["alpha"], inp["xi"], inp["zeta"],
-                                      inp["kappa"], inp.get("mask"),
-                                      v_o.reshape(w.T, -1)).reshape(v_o.shape)
-    v_tol = V_ATOL + V_RTOL * np.abs(v_o) + v_extra
-    first = first_ambiguous_step(v_o, w.theta, v_tol)       # [B, N]
+    if allowance:
+        v_extra = soma_rounding_allowance(w, xk, chan, mrow, inp["alpha"], inp["xi"],
+                                          inp["zeta"], inp["kappa"], inp.get("mask"),
+                                          v_o.reshape(w.T, -1)).reshape(v_o.shape)
+        v_tol = V_ATOL + V_RTOL * np.abs(v_o) + v_extra
+        first = first_ambiguous_step(v_o, w.theta, v_tol)       # [B, N]
+    else:
+        v_extra = 0.0
+        first = first_ambiguous_step(v_o, w.theta)
     amb = first < w.T
     gs = inp["gs"].clone()
     gs[:, torch.from_numpy(amb)] = 0
@@ -223,11 +249,13 @@ def check_layer(w, seed_inputs=None, with_gv=True):
     dev = to_dev(inp)
     got = run_gpu(w, dev, gs.cuda(), None if gv is None else gv.cuda())
     ref = oracle.backward_layer(w, dict(inp, gv=gv), gs=gs, want_dvs=True)
-    extra = direction_rounding_allowance(
-        w, xk, chan, mrow, inp["alpha"], inp["xi"], inp["zeta"],
-        inp["kappa"], inp.get("mask"), ref["dvs"].reshape(w.T, w.B * w.N))
-    if not np.isscalar(extra):
-        extra = oracle.layer_gx(w, extra)
+    extra = 0.0
+    if allowance:
+        extra = direction_rounding_allowance(
+            w, xk, chan, mrow, inp["alpha"], inp["xi"], inp["zeta"],
+            inp["kappa"], inp.get("mask"), ref["dvs"].reshape(w.T, w.B * w.N))
+        if not np.isscalar(extra):
+            extra = oracle.layer_gx(w, extra)
 
     t_idx = np.arange(w.T)[:, None, None]
     v_mask = t_idx <= first[None]                           # V compared up to the first ambiguous step
@@ -236,11 +264,13 @@ def check_layer(w, seed_inputs=None, with_gv=True):
     assert np.array_equal(got["s"][s_mask], s_o[s_mask]), \
         f"spikes differ at {int((got['s'][s_mask] != s_o[s_mask]).sum())} unambiguous steps"
     assert set(np.unique(got["s"]).tolist()) <= {0.0, 1.0}
-    if w.dtype == "bf16":
-        assert_close("grad_x", got["gx"], ref["gx"], BF16_RTOL, BF16_ATOL_REL, atol_abs=extra)
+    if allowance:
+        gx_rel = BF16_ATOL_REL if w.dtype == "bf16" else gx_atol_rel(w, inp["alpha"])
+        p_rel = G_ATOL_REL
     else:
-        assert_close("grad_x", got["gx"], ref["gx"], G_RTOL, gx_atol_rel(w, inp["alpha"]),
-                     atol_abs=extra)
+        gx_rel, p_rel = GX_ATOL_REL, P_ATOL_REL
+    assert_close("grad_x", got["gx"], ref["gx"], BF16_RTOL if w.dtype == "bf16" else G_RTOL,
+                 gx_rel, atol_abs=extra)
     for k in ("galpha", "gxi", "gzeta", "gkappa", "gbeta"):
-        assert_close(k, got[k], ref[k], G_RTOL, G_ATOL_REL)
+        assert_close(k, got[k], ref[k], G_RTOL, p_rel)
     return dict(ambiguous_neurons=int(amb.sum()), spikes=float(s_o.mean()))

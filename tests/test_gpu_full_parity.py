@@ -1,0 +1,50 @@
+"""Every neuron of each full-size layer workload against the oracle, at the stated bounds.
+
+The five layer shapes (tiny, conv, deeper bf16 conv, event-stream, transformer token with
+per-neuron branch gating) run at their full sizes in the benchmark's launch configuration;
+the oracle simulates every neuron on all host cores (tests/full_parity.py). No rounding
+allowance is added: V^s within 1e-6 + 1e-5|v|, spikes identical outside the 1e-5 window,
+float32 gradients within 1e-4 relative + 1e-6 RMS, bfloat16 dL/dX within 2e-2 relative
++ 1e-6 RMS, parameter gradients against the float64 sums over the whole layer.
+
+With DENDSN_PARITY_REPORT set to a directory, each case also writes its report there
+(worst error over bound per quantity, ambiguous-neuron count, timings).
+"""
+import json
+import os
+
+import pytest
+import torch
+
+import oracle
+from paper_2412_06355_gb300 import binding
+from paper_2412_06355_gb300.workloads import WORKLOADS
+
+import full_parity
+
+pytestmark = pytest.mark.gpu
+
+LAYERS = ["tiny", "conv", "deepconv_bf16", "event", "token_dbg"]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.fail("these tests need a CUDA device")
+    binding.load()
+    oracle.build()
+
+
+@pytest.mark.parametrize("name", LAYERS)
+def test_full_layer_every_neuron(name):
+    w = WORKLOADS[name]
+    rep = full_parity.run(w)
+    out = os.environ.get("DENDSN_PARITY_REPORT")
+    if out:
+        os.makedirs(out, exist_ok=True)
+        with open(os.path.join(out, f"full_{name}.json"), "w") as f:
+            json.dump(rep, f, indent=1)
+    print(json.dumps(rep))
+    bad = full_parity.failures(rep)
+    assert not bad, f"{name}: " + "; ".join(bad)
+    assert rep["spike_rate"] > 0.0

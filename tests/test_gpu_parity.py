@@ -18,9 +18,10 @@ import oracle
 from paper_2412_06355_gb300 import binding, workloads
 from paper_2412_06355_gb300.workloads import WORKLOADS, scaled
 
-from parity import (BF16_ATOL_REL, BF16_RTOL, G_ATOL_REL, G_RTOL, V_ATOL, V_RTOL,
-                    assert_close, check_layer, direction_rounding_allowance,
-                    first_ambiguous_step, gx_atol_rel, soma_rounding_allowance, to_dev)
+from parity import (BF16_ATOL_REL, BF16_RTOL, G_ATOL_REL, G_RTOL, GX_ATOL_REL, P_ATOL_REL,
+                    V_ATOL, V_RTOL, assert_close, check_layer, direction_rounding_allowance,
+                    first_ambiguous_step, gx_atol_rel, needs_allowance,
+                    soma_rounding_allowance, to_dev)
 
 pytestmark = pytest.mark.gpu
 
@@ -286,6 +287,7 @@ BIG = workloads.Workload("offsets_beyond_int32", T=64, B=65, N=131072, K=4, G=1,
                          ["offsets_beyond_int32"])
 def test_full_size_sampled(name, kw):
     w = (BIG if name == BIG.name else WORKLOADS[name]).with_(**kw)
+    allow = needs_allowance(w)
     cfg = binding.config_of(w)
     inp = workloads.make_inputs(w, "cuda")          # full size, generated on the device
     b_idx, n_idx = sample_neurons(w, 3000, seed=w.seed)
@@ -301,8 +303,10 @@ def test_full_size_sampled(name, kw):
     prm = [inp[k].cpu() for k in ("alpha", "xi", "zeta", "kappa")]
     mask = None if inp["mask"] is None else inp["mask"].cpu()
     s_o, v_o = oracle.forward(ocfg, xs, chan, mrow, *prm, mask)
-    v_extra = soma_rounding_allowance(w, oracle.to_f64(xs), chan, mrow, *prm, mask, v_o)
-    first = first_ambiguous_step(v_o, w.theta, V_ATOL + V_RTOL * np.abs(v_o) + v_extra)
+    v_extra = (soma_rounding_allowance(w, oracle.to_f64(xs), chan, mrow, *prm, mask, v_o)
+               if allow else 0.0)
+    first = (first_ambiguous_step(v_o, w.theta, V_ATOL + V_RTOL * np.abs(v_o) + v_extra)
+             if allow else first_ambiguous_step(v_o, w.theta))
     keep = first == w.T
 
     # upstream gradient: zero except on the unambiguous sampled neurons
@@ -327,13 +331,17 @@ def test_full_size_sampled(name, kw):
 
     ref = oracle.backward(ocfg, xs, chan, mrow, *prm, mask, gs_sample[:, bt, nt].cpu(),
                           want_dvs=True)
-    extra = direction_rounding_allowance(w, oracle.to_f64(xs), chan, mrow, *prm, mask,
-                                         ref["dvs"])
-    rt, ar = ((BF16_RTOL, BF16_ATOL_REL) if w.dtype == "bf16"
-              else (G_RTOL, gx_atol_rel(w, inp["alpha"])))
+    rt = BF16_RTOL if w.dtype == "bf16" else G_RTOL
+    if allow:
+        extra = direction_rounding_allowance(w, oracle.to_f64(xs), chan, mrow, *prm, mask,
+                                             ref["dvs"])
+        ar = BF16_ATOL_REL if w.dtype == "bf16" else gx_atol_rel(w, inp["alpha"])
+        p_rel = G_ATOL_REL
+    else:
+        extra, ar, p_rel = 0.0, GX_ATOL_REL, P_ATOL_REL
     assert_close("grad_x", got_gx, ref["gx"], rt, ar, atol_abs=extra)
     for k in ("galpha", "gxi", "gzeta", "gkappa", "gbeta"):
-        assert_close(k, oracle.to_f64(g[k]), ref[k], G_RTOL, G_ATOL_REL)
+        assert_close(k, oracle.to_f64(g[k]), ref[k], G_RTOL, p_rel)
     # every non-sampled neuron received zero upstream gradient: its grad_x is zero
     gx = g["gx"]
     if w.layout == "paper":
