@@ -47,6 +47,40 @@ cudaError_t launch_finalize(const FinArgs &a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+namespace {
+struct ResidentKey {
+    const void *kernel;
+    int threads;
+    size_t bytes;
+    int device;
+    int blocks;
+};
+std::mutex g_resident_mutex;
+ResidentKey g_resident[256];
+int g_resident_n = 0;
+}  // namespace
+
+cudaError_t resident_blocks(const void *kernel, int threads, size_t bytes, int *out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(g_resident_mutex);
+    for (int i = 0; i < g_resident_n; ++i) {
+        const ResidentKey &k = g_resident[i];
+        if (k.kernel == kernel && k.threads == threads && k.bytes == bytes && k.device == dev) {
+            *out = k.blocks;
+            return cudaSuccess;
+        }
+    }
+    int n = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, threads, bytes);
+    if (e != cudaSuccess) return e;
+    if (g_resident_n < (int)(sizeof g_resident / sizeof g_resident[0]))
+        g_resident[g_resident_n++] = ResidentKey{kernel, threads, bytes, dev, n};
+    *out = n;
+    return cudaSuccess;
+}
+
 }  // namespace dendsn
 
 using namespace dendsn;
@@ -90,30 +124,82 @@ int sm_count() {
 
 bool is01(int32_t v) { return v == 0 || v == 1; }
 
-// Tiling of the O x P neuron matrix for blocks of nt threads, lpn lanes per neuron, about
-// per_sm blocks per SM in total (fewer means more rows per thread).
-dendsn_status tile(Geometry &g, int nt, int lpn, int64_t sms, int per_sm, int64_t *blocks) {
+// Column tiling of the O x P neuron matrix for blocks of nt threads with lpn lanes per
+// neuron: TXn columns x TY row lanes per block.
+void tile_columns(Geometry &g, int nt, int lpn) {
     const int W = 32 / lpn;                     // columns per warp
     const int full = nt / lpn;                  // columns of a one-row tile
     g.TXn = (g.inner >= W && g.P % full == 0) ? full : W;
     g.TY = nt / (g.TXn * lpn);
     g.seg = (g.inner % W == 0) ? W : ((W % g.inner == 0) ? g.inner : 1);
     g.nCT = (int32_t)((g.P + g.TXn - 1) / g.TXn);
-    // rows per thread: about per_sm blocks per SM in total, at least one row
-    const int64_t target_blocks = (int64_t)per_sm * sms;
-    const int64_t rg_target = std::max<int64_t>(1, (target_blocks + g.nCT - 1) / g.nCT);
-    const int64_t rows_per_rg = std::max<int64_t>(1, (g.O + rg_target - 1) / rg_target);
-    g.R = (int32_t)std::max<int64_t>(1, (rows_per_rg + g.TY - 1) / g.TY);
-    const int64_t nRG = (g.O + (int64_t)g.R * g.TY - 1) / ((int64_t)g.R * g.TY);
-    g.nRG = (int32_t)nRG;
     // channels one column tile touches (tiles start at multiples of TXn)
     if (g.TXn % g.inner == 0) g.nch_max = g.TXn / g.inner;
     else if (g.inner % g.TXn == 0) g.nch_max = 1;
     else g.nch_max = std::min<int32_t>(g.C, (g.TXn - 1) / g.inner + 2);
-    *blocks = (int64_t)g.nCT * nRG;
+}
+
+// Row tiling: R rows per thread and nRG row groups, so that the grid is nCT * nRG blocks.
+// The fixed sizing aims at about per_sm blocks per SM (measured best on the layer
+// workloads when a wave is nearly full). With `resident` blocks of the kernel fitting on
+// one SM the grid runs in waves of resident * sms blocks, and a last wave that is only
+// partly filled leaves SMs idle while it finishes: the time is modelled as
+// (waves) x (rows per thread + one row's worth of per-block set-up and reduction), and the
+// row groups that minimise it (over up to four times the waves of the fixed sizing)
+// replace the fixed sizing when the model predicts at least 8% less time. Below that the
+// model is within its own error: on the layer workloads it predicted 4-6% that did not
+// materialise, while its 11-20% predictions gave 7-13% (token layer forward and backward,
+// event-stream layer backward).
+dendsn_status tile_rows(Geometry &g, int64_t sms, int resident, int per_sm, int64_t *blocks) {
+    const int64_t rows = std::max<int64_t>(1, (g.O + g.TY - 1) / g.TY);   // row slots per column
+    auto rows_for = [&](int64_t nrg, int64_t *nrg_used) {
+        const int64_t R = std::max<int64_t>(1, (rows + nrg - 1) / nrg);
+        *nrg_used = (rows + R - 1) / R;
+        return R;
+    };
+    // the fixed sizing: about per_sm blocks per SM in total, at least one row
+    const int64_t target_blocks = (int64_t)per_sm * sms;
+    const int64_t rg_target = std::max<int64_t>(1, (target_blocks + g.nCT - 1) / g.nCT);
+    int64_t best_n = 0;
+    int64_t best_R = rows_for(rg_target, &best_n);
+    if (resident > 0) {
+        const int64_t cap = (int64_t)resident * sms;
+        auto cost = [&](int64_t nrg, int64_t R) {
+            return (double)((g.nCT * nrg + cap - 1) / cap) * (double)(R + 1);
+        };
+        const double fixed_cost = cost(best_n, best_R);
+        const int64_t wmax = std::min<int64_t>(64, 4 * std::max<int64_t>(1, (target_blocks + cap - 1) / cap));
+        double best_cost = 0.0;
+        int64_t cand_R = 0, cand_n = 0;
+        for (int64_t w = 1; w <= wmax; ++w) {
+            const int64_t top = std::max<int64_t>(1, std::min<int64_t>(rows, w * cap / g.nCT));
+            for (int64_t nrg = std::max<int64_t>(1, top - 2); nrg <= top; ++nrg) {
+                int64_t used = 0;
+                const int64_t R = rows_for(nrg, &used);
+                const double c = cost(used, R);
+                if (cand_n == 0 || c < best_cost || (c == best_cost && used < cand_n)) {
+                    best_cost = c;
+                    cand_R = R;
+                    cand_n = used;
+                }
+            }
+        }
+        if (cand_n > 0 && best_cost < 0.92 * fixed_cost) {
+            best_R = cand_R;
+            best_n = cand_n;
+        }
+    }
+    g.R = (int32_t)best_R;
+    g.nRG = (int32_t)((g.O + (int64_t)g.R * g.TY - 1) / ((int64_t)g.R * g.TY));
+    *blocks = (int64_t)g.nCT * g.nRG;
     if (*blocks > INT32_MAX) return fail(DENDSN_ERR_UNSUPPORTED, "grid too large");
     return DENDSN_OK;
 }
+
+cudaError_t dispatch_forward(const dendsn_config &cfg, int layout, const FwdArgs &a, int blocks,
+                             cudaStream_t s, int *resident = nullptr);
+cudaError_t dispatch_backward(const dendsn_config &cfg, int layout, int L, const BwdArgs &a,
+                              int blocks, cudaStream_t s, int *resident = nullptr);
 
 dendsn_status make_plan(const dendsn_config *cfg, Plan *pl) {
     if (cfg == nullptr) return fail(DENDSN_ERR_INVALID_ARG, "cfg is NULL");
@@ -164,22 +250,49 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl) {
     pl->gf = g;
     pl->gb = g;
     const int KTB = bwd_lane_compartments(c.K, c.G, c.x_dtype, g.L);
-    dendsn_status st = tile(pl->gf, fwd_threads(c.K), c.K / KT, sms, 16, &bf);
-    if (st != DENDSN_OK) return st;
-    // backward: when every column is its own channel (inner = 1) each thread's parameter
-    // setup is heavier, and twice the rows per thread measured faster (token layer 285 ->
-    // 272 us); elsewhere 16 blocks per SM measured best
-    const int bwd_per_sm = (c.inner == 1) ? 8 : 16;
-    if ((st = tile(pl->gb, bwd_threads(KTB), c.K / KTB, sms, bwd_per_sm, &bb)) != DENDSN_OK) return st;
-    pl->blocks_f = (int)bf;
-    pl->blocks_b = (int)bb;
+    tile_columns(pl->gf, fwd_threads(c.K), c.K / KT);
+    tile_columns(pl->gb, bwd_threads(KTB), c.K / KTB);
     pl->sx = (c.x_dtype == DENDSN_BF16) ? 2 : 4;
     pl->layout = (c.K > 1 && c.inner > 1) ? c.layout : 0;   // otherwise the layouts coincide
+    // narrow layers with long horizons: one warp per neuron, time scanned in parallel
+    pl->tp = c.T >= kTpMinT && BN <= kTpMaxNeurons && tp_smem_bytes(c.T, c.K, true) <= kTpMaxSmem;
+    // blocks of the forward and backward kernels that fit on one SM. The backward's is taken
+    // for the compartments-innermost layout and the build without dL/dbeta, so that both
+    // layouts and both builds of a layer share one tiling (and sum the parameter gradients
+    // in the same order).
+    int res_f = 0, res_b = 0;
+    if (!pl->tp && O > 0 && c.T > 0) {
+        FwdArgs fa;
+        std::memset(&fa, 0, sizeof fa);
+        fa.g = pl->gf;
+        fa.p.mask_mode = c.mask_per_neuron ? 2 : 0;
+        BwdArgs ba;
+        std::memset(&ba, 0, sizeof ba);
+        ba.g = pl->gb;
+        ba.p.mask_mode = fa.p.mask_mode;
+        ba.p.residual = c.residual;
+        // a failed query (no device) leaves the residency unknown: the fixed sizing applies
+        if (dispatch_forward(c, pl->layout, fa, 0, nullptr, &res_f) != cudaSuccess) {
+            res_f = 0;
+            (void)cudaGetLastError();
+        }
+        if (dispatch_backward(c, 0, g.L, ba, 0, nullptr, &res_b) != cudaSuccess) {
+            res_b = 0;
+            (void)cudaGetLastError();
+        }
+    }
+    dendsn_status st = tile_rows(pl->gf, sms, res_f, 16, &bf);
+    if (st != DENDSN_OK) return st;
+    // backward without the residency: when every column is its own channel (inner = 1)
+    // each thread's parameter setup is heavier, and twice the rows per thread measured
+    // faster (token layer 285 -> 272 us); elsewhere 16 blocks per SM measured best
+    const int bwd_per_sm = (c.inner == 1) ? 8 : 16;
+    if ((st = tile_rows(pl->gb, sms, res_b, bwd_per_sm, &bb)) != DENDSN_OK) return st;
+    pl->blocks_f = (int)bf;
+    pl->blocks_b = (int)bb;
     const size_t NP = 2 * (size_t)c.K + 2 * (size_t)g.Kb + 1;     // + the beta slot
     pl->scratch_bytes = (size_t)bb * pl->gb.nch_max * NP * sizeof(float);
     pl->scratch_bytes = (pl->scratch_bytes + 15) / 16 * 16;
-    // narrow layers with long horizons: one warp per neuron, time scanned in parallel
-    pl->tp = c.T >= kTpMinT && BN <= kTpMaxNeurons && tp_smem_bytes(c.T, c.K, true) <= kTpMaxSmem;
     if (pl->tp) {
         pl->gf.n_ck = pl->gb.n_ck = 0;                 // the backward recomputes from x alone
         pl->scratch_bytes = ((size_t)BN * NP * sizeof(float) + 15) / 16 * 16;
@@ -223,34 +336,34 @@ dendsn_status check_params(const float *alpha, const float *xi, const float *zet
 #define DENDSN_FWD_CASE(KK, GG)                                                         \
     if (cfg.K == KK && cfg.G == GG) {                                                   \
         switch ((cfg.psi * 2 + cfg.x_dtype) * 2 + layout) {                             \
-        case 0: return launch_forward<KK, GG, 0, 0, 0>(a, blocks, s);                   \
-        case 1: return launch_forward<KK, GG, 0, 0, 1>(a, blocks, s);                   \
-        case 2: return launch_forward<KK, GG, 0, 1, 0>(a, blocks, s);                   \
-        case 3: return launch_forward<KK, GG, 0, 1, 1>(a, blocks, s);                   \
-        case 4: return launch_forward<KK, GG, 1, 0, 0>(a, blocks, s);                   \
-        case 5: return launch_forward<KK, GG, 1, 0, 1>(a, blocks, s);                   \
-        case 6: return launch_forward<KK, GG, 1, 1, 0>(a, blocks, s);                   \
-        default: return launch_forward<KK, GG, 1, 1, 1>(a, blocks, s);                  \
+        case 0: return launch_forward<KK, GG, 0, 0, 0>(a, blocks, s, resident);         \
+        case 1: return launch_forward<KK, GG, 0, 0, 1>(a, blocks, s, resident);         \
+        case 2: return launch_forward<KK, GG, 0, 1, 0>(a, blocks, s, resident);         \
+        case 3: return launch_forward<KK, GG, 0, 1, 1>(a, blocks, s, resident);         \
+        case 4: return launch_forward<KK, GG, 1, 0, 0>(a, blocks, s, resident);         \
+        case 5: return launch_forward<KK, GG, 1, 0, 1>(a, blocks, s, resident);         \
+        case 6: return launch_forward<KK, GG, 1, 1, 0>(a, blocks, s, resident);         \
+        default: return launch_forward<KK, GG, 1, 1, 1>(a, blocks, s, resident);        \
         }                                                                               \
     }
 
 // layout: 0 compartments innermost, 1 the paper's layer layout (0 when K = 1 or inner = 1: the same)
 cudaError_t dispatch_forward(const dendsn_config &cfg, int layout, const FwdArgs &a, int blocks,
-                             cudaStream_t s) {
+                             cudaStream_t s, int *resident) {
     DENDSN_KG_LIST(DENDSN_FWD_CASE)
     return cudaErrorInvalidValue;
 }
 
 #define DENDSN_BWD_L(KK, GG, LL)                                                        \
     switch ((cfg.psi * 2 + cfg.x_dtype) * 2 + layout) {                                 \
-    case 0: return launch_backward<KK, GG, 0, 0, LL, 0>(a, blocks, s);                  \
-    case 1: return launch_backward<KK, GG, 0, 0, LL, 1>(a, blocks, s);                  \
-    case 2: return launch_backward<KK, GG, 0, 1, LL, 0>(a, blocks, s);                  \
-    case 3: return launch_backward<KK, GG, 0, 1, LL, 1>(a, blocks, s);                  \
-    case 4: return launch_backward<KK, GG, 1, 0, LL, 0>(a, blocks, s);                  \
-    case 5: return launch_backward<KK, GG, 1, 0, LL, 1>(a, blocks, s);                  \
-    case 6: return launch_backward<KK, GG, 1, 1, LL, 0>(a, blocks, s);                  \
-    default: return launch_backward<KK, GG, 1, 1, LL, 1>(a, blocks, s);                 \
+    case 0: return launch_backward<KK, GG, 0, 0, LL, 0>(a, blocks, s, resident);        \
+    case 1: return launch_backward<KK, GG, 0, 0, LL, 1>(a, blocks, s, resident);        \
+    case 2: return launch_backward<KK, GG, 0, 1, LL, 0>(a, blocks, s, resident);        \
+    case 3: return launch_backward<KK, GG, 0, 1, LL, 1>(a, blocks, s, resident);        \
+    case 4: return launch_backward<KK, GG, 1, 0, LL, 0>(a, blocks, s, resident);        \
+    case 5: return launch_backward<KK, GG, 1, 0, LL, 1>(a, blocks, s, resident);        \
+    case 6: return launch_backward<KK, GG, 1, 1, LL, 0>(a, blocks, s, resident);        \
+    default: return launch_backward<KK, GG, 1, 1, LL, 1>(a, blocks, s, resident);       \
     }
 
 #define DENDSN_BWD_CASE(KK, GG)                                                         \
@@ -260,7 +373,7 @@ cudaError_t dispatch_forward(const dendsn_config &cfg, int layout, const FwdArgs
     }
 
 cudaError_t dispatch_backward(const dendsn_config &cfg, int layout, int L, const BwdArgs &a,
-                              int blocks, cudaStream_t s) {
+                              int blocks, cudaStream_t s, int *resident) {
     DENDSN_KG_LIST(DENDSN_BWD_CASE)
     return cudaErrorInvalidValue;
 }

@@ -313,7 +313,7 @@ struct PairArith {
     static constexpr int KTb = KT;
     struct LP { float2 a[N2], nxi[N2], iz[N2], km[N2], lm[N2]; };
     struct St { float2 v[N2]; };
-    struct Acc { float2 ga[N2], ngxi[N2], ngz[N2], gk[N2]; };   // ngxi, ngz: negated sums
+    struct Acc { float2 ga[N2], ngxi[N2], ngz[N2], ngk[N2]; };  // ngxi, ngz, ngk: negated sums
     // mask value as the engine keeps it (see above)
     static __device__ __forceinline__ float mask_term(float m) {
         if constexpr (PSI == PSI_MEXHAT) return m != 0.f ? 0.f : -INFINITY;
@@ -423,7 +423,32 @@ struct PairArith {
     }
     static __device__ __forceinline__ void acc_zero(Acc &c) {
 #pragma unroll
-        for (int m = 0; m < N2; ++m) { c.ga[m] = f2(0.f); c.ngxi[m] = f2(0.f); c.ngz[m] = f2(0.f); c.gk[m] = f2(0.f); }
+        for (int m = 0; m < N2; ++m) { c.ga[m] = f2(0.f); c.ngxi[m] = f2(0.f); c.ngz[m] = f2(0.f); c.ngk[m] = f2(0.f); }
+    }
+    // Floats in Acc; acc_flush adds them into per-thread totals t[q * NT] and zeroes them,
+    // acc_load reads them back.
+    static constexpr int kAccFloats = 8 * N2;
+    template <int NT>
+    static __device__ __forceinline__ void acc_flush(Acc &c, float *t) {
+#pragma unroll
+        for (int m = 0; m < N2; ++m) {
+            const float2 *f[4] = {&c.ga[m], &c.ngxi[m], &c.ngz[m], &c.ngk[m]};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                t[(8 * m + 2 * q) * NT] = __fadd_rn(t[(8 * m + 2 * q) * NT], f[q]->x);
+                t[(8 * m + 2 * q + 1) * NT] = __fadd_rn(t[(8 * m + 2 * q + 1) * NT], f[q]->y);
+            }
+        }
+        acc_zero(c);
+    }
+    template <int NT>
+    static __device__ __forceinline__ void acc_load(Acc &c, const float *t) {
+#pragma unroll
+        for (int m = 0; m < N2; ++m) {
+            float2 *f[4] = {&c.ga[m], &c.ngxi[m], &c.ngz[m], &c.ngk[m]};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) *f[q] = make_float2(t[(8 * m + 2 * q) * NT], t[(8 * m + 2 * q + 1) * NT]);
+        }
     }
     // [alpha KT | xi KT | zeta KTb | kappa KTb]; the first three carry the factor 1/zeta here
     static __device__ __forceinline__ void acc_export(const LP &lp, const Acc &c, float *v) {
@@ -435,7 +460,7 @@ struct PairArith {
             v[2 * m] = ga.x;                     v[2 * m + 1] = ga.y;
             v[KT + 2 * m] = -gxi.x;              v[KT + 2 * m + 1] = -gxi.y;
             v[2 * KT + 2 * m] = -gz.x;           v[2 * KT + 2 * m + 1] = -gz.y;
-            v[3 * KT + 2 * m] = c.gk[m].x;       v[3 * KT + 2 * m + 1] = c.gk[m].y;
+            v[3 * KT + 2 * m] = -c.ngk[m].x;     v[3 * KT + 2 * m + 1] = -c.ngk[m].y;
         }
     }
     // One reverse step: V^d[t] (vdt), V^d[t-1] (vdp) and dL/dZ[t] (dz) update the scaled
@@ -446,37 +471,40 @@ struct PairArith {
     // dL/dV^d is dL/du / zeta; du/dxi = -1/zeta; du/dzeta = -u / zeta.
     static __device__ __forceinline__ void backward(const LP &lp, const St &vdt, const St &vdp, float dz,
                                                     St &Ad, Acc &acc, float res, float (&gx)[KT]) {
-        const float2 dz2 = f2(dz);
+        const float2 ndz2 = f2(-dz);
         const float2 res2 = f2(res);
 #pragma unroll
         for (int m = 0; m < N2; ++m) {
-            const float2 g = pair_back(lp, m, vdt.v[m], vdp.v[m], dz2, res2, Ad.v[m], acc);
+            const float2 g = pair_back(lp, m, vdt.v[m], vdp.v[m], ndz2, res2, Ad.v[m], acc);
             gx[2 * m] = g.x;
             gx[2 * m + 1] = g.y;
         }
     }
-    // Pair m of one reverse step (see backward); returns dL/dX[t] of the pair.
+    // Pair m of one reverse step (see backward), given ndz2 = -dL/dZ[t]; returns dL/dX[t]
+    // of the pair.
     static __device__ __forceinline__ float2 pair_back(const LP &lp, int m, float2 vdt, float2 vdp,
-                                                       float2 dz2, float2 res2, float2 &Adm, Acc &acc) {
+                                                       float2 ndz2, float2 res2, float2 &Adm, Acc &acc) {
         {
             const float2 u = ffma2(vdt, lp.iz[m], lp.nxi[m]);
-            const float2 gy = fmul2(lp.km[m], dz2);              // dL/dY
+            const float2 ngy = fmul2(lp.km[m], ndz2);            // -dL/dY
             float2 y, du;                                        // m Y, dL/du
             if constexpr (PSI == PSI_MEXHAT) {
                 const float2 ss = fmul2(u, u);
                 const float2 t = ffma2(f2(kNegHalfLog2e), ss, lp.lm[m]);
                 const float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
                 y = ffma2(neg2(ss), e, e);
-                const float2 w = fmul2(fadd2(ss, f2(-3.f)), e);  // psi'(r) / r
-                du = fmul2(fmul2(w, u), gy);
+                // psi'(r) / r = (r^2 - 3) e^{-r^2/2} = -(2 e^{-r^2/2} + psi(r)): one fused
+                // multiply-add from y; its sign cancels against that of -dL/dY
+                const float2 nw = ffma2(f2(2.f), e, y);
+                du = fmul2(nw, fmul2(u, ngy));
             } else {
                 y = fmul2(lp.lm[m], make_float2(fabsf(u.x), fabsf(u.y)));
-                du = make_float2(u.x > 0.f ? gy.x : (u.x < 0.f ? -gy.x : 0.f),
-                                 u.y > 0.f ? gy.y : (u.y < 0.f ? -gy.y : 0.f));
+                du = make_float2(u.x > 0.f ? -ngy.x : (u.x < 0.f ? ngy.x : 0.f),
+                                 u.y > 0.f ? -ngy.y : (u.y < 0.f ? ngy.y : 0.f));
             }
             acc.ngxi[m] = fadd2(acc.ngxi[m], du);                // zeta dxi = -sum du
             acc.ngz[m] = ffma2(u, du, acc.ngz[m]);               // zeta dzeta = -sum u du
-            acc.gk[m] = ffma2(y, dz2, acc.gk[m]);                // dkappa = sum m Y dz
+            acc.ngk[m] = ffma2(y, ndz2, acc.ngk[m]);             // dkappa = sum m Y dz
             Adm = ffma2(lp.a[m], Adm, du);
             acc.ga[m] = ffma2(Adm, vdp, acc.ga[m]);              // zeta dalpha
             return ffma2(Adm, lp.iz[m], res2);
@@ -554,6 +582,30 @@ struct ScalarArith {
         for (int i = 0; i < KT; ++i) { c.ga[i] = 0.f; c.gxi[i] = 0.f; }
 #pragma unroll
         for (int b = 0; b < KTb; ++b) { c.gz[b] = 0.f; c.gk[b] = 0.f; }
+    }
+    // Floats in Acc; acc_flush adds them into per-thread totals t[q * NT] and zeroes them,
+    // acc_load reads them back.
+    static constexpr int kAccFloats = 2 * KT + 2 * KTb;
+    template <int NT>
+    static __device__ __forceinline__ void acc_flush(Acc &c, float *t) {
+#pragma unroll
+        for (int i = 0; i < KT; ++i) {
+            t[i * NT] = __fadd_rn(t[i * NT], c.ga[i]);
+            t[(KT + i) * NT] = __fadd_rn(t[(KT + i) * NT], c.gxi[i]);
+        }
+#pragma unroll
+        for (int b = 0; b < KTb; ++b) {
+            t[(2 * KT + b) * NT] = __fadd_rn(t[(2 * KT + b) * NT], c.gz[b]);
+            t[(2 * KT + KTb + b) * NT] = __fadd_rn(t[(2 * KT + KTb + b) * NT], c.gk[b]);
+        }
+        acc_zero(c);
+    }
+    template <int NT>
+    static __device__ __forceinline__ void acc_load(Acc &c, const float *t) {
+#pragma unroll
+        for (int i = 0; i < KT; ++i) { c.ga[i] = t[i * NT]; c.gxi[i] = t[(KT + i) * NT]; }
+#pragma unroll
+        for (int b = 0; b < KTb; ++b) { c.gz[b] = t[(2 * KT + b) * NT]; c.gk[b] = t[(2 * KT + KTb + b) * NT]; }
     }
     static __device__ __forceinline__ void acc_export(const LP &, const Acc &c, float *v) {
 #pragma unroll
@@ -1205,15 +1257,23 @@ dendsn_forward_staged_kernel(const FwdArgs A) {
 }
 
 // ---------------------------------------------------------------- backward
+// Rows of the reduction buffer are NT + 1 floats apart, so that the threads of a warp that
+// read one entry of consecutive gradient slots hit consecutive banks (rows NT apart would
+// put all of them in one bank).
+template <int NT> constexpr int red_stride() { return NT + 1; }
+// Bytes of shared memory block_partials needs for NA1 gradient slots.
+constexpr size_t red_bytes(int NA1, int NT) { return sizeof(float) * (size_t)NA1 * (NT + 1); }
+
 // Per-channel partial sums of a block's parameter-gradient vectors v (one per thread,
 // [alpha KT | xi KT | zeta KTb | kappa KTb | beta]) in a fixed order: segmented warp
 // shuffles over the columns of one channel, then the run leaders in shared memory (red,
-// NA1 * NT floats), one partial per (block, channel) to `partials`.
+// red_bytes(NA1, NT)), one partial per (block, channel) to `partials`.
 template <int KT, int G, int LPN, int NT, int NA1>
 __device__ __forceinline__ void block_partials(const Geometry &g, const ThreadPos &pos,
                                                float (&v)[NA1], float *red, float *partials) {
     constexpr int KTb = KT / G;
     constexpr int NA = NA1 - 1;
+    constexpr int RS = red_stride<NT>();
     // stage 1: within a warp, columns of one channel come in aligned runs of g.seg
     for (int d = 1; d < g.seg; d <<= 1) {
 #pragma unroll
@@ -1223,7 +1283,7 @@ __device__ __forceinline__ void block_partials(const Geometry &g, const ThreadPo
     // stage 2: run leaders meet in shared memory; red[a][tid] (reuses the history space)
     __syncthreads();
 #pragma unroll
-    for (int a = 0; a < NA1; ++a) red[a * NT + threadIdx.x] = v[a];
+    for (int a = 0; a < NA1; ++a) red[a * RS + threadIdx.x] = v[a];
     __syncthreads();
     const int ct = blockIdx.x % g.nCT;
     const int p0 = ct * g.TXn;
@@ -1244,7 +1304,7 @@ __device__ __forceinline__ void block_partials(const Geometry &g, const ThreadPo
         float sum = 0.f;
         for (int ry = 0; ry < g.TY; ++ry)
             for (int cx = cx_lo; cx < cx_hi; cx += g.seg)
-                sum = __fadd_rn(sum, red[a * NT + (ry * g.TXn + cx) * LPN + sub]);
+                sum = __fadd_rn(sum, red[a * RS + (ry * g.TXn + cx) * LPN + sub]);
         int slot;
         if (a < KT) slot = sub * KT + a;                                        // alpha
         else if (a < 2 * KT) slot = g.K + sub * KT + (a - KT);                  // xi
@@ -1257,6 +1317,14 @@ __device__ __forceinline__ void block_partials(const Geometry &g, const ThreadPo
 
 template <int KT, int G>
 constexpr int acc_count() { return 2 * KT + 2 * (KT / G); }
+
+// Whether the chunked backward keeps two-level parameter-gradient sums for rows of several
+// chunks (L == 8): all builds but eight float32 compartments per lane, whose totals would
+// take the shared memory of one of their three resident blocks per SM.
+template <int K, int G, typename XT, int L>
+constexpr bool row_totals() {
+    return L > 4 && !(bwd_lane_compartments(K, G, xt_code<XT>(), L) >= 8 && std::is_same<XT, float>::value);
+}
 
 // BETA: also accumulate dL/dbeta (a learnable somatic decay); a separate instance because
 // even one more live accumulator slows the register-history path measurably.
@@ -1323,6 +1391,17 @@ dendsn_backward_kernel(const BwdArgs A) {
     HistRaw *hist = reinterpret_cast<HistRaw *>(sregion);                             // [L][NT]
     float *hist_vs = reinterpret_cast<float *>(hist + (SHIST ? L * NT : 0));   // [L][NT]
     XRaw *xring = reinterpret_cast<XRaw *>(hist_vs + (SHIST ? L * NT : 0)) + threadIdx.x;   // [D][NT]
+    // rows of several chunks: the parameter-gradient terms of each row are summed on their
+    // own and the row sums added into per-thread totals [kAccFloats + 1][NT] after the x ring
+    // (a two-level sum: float32 rounding grows with the terms of one row, not of all rows)
+    constexpr bool TOTALS = row_totals<K, G, XT, L>();
+    float *const tot = reinterpret_cast<float *>(reinterpret_cast<char *>(hist_vs + (SHIST ? L * NT : 0)) +
+                                                 (BASYNC ? sizeof(XRaw) * D * NT : 0)) + threadIdx.x;
+    const bool use_tot = TOTALS && nc > 1;
+    if (use_tot) {
+#pragma unroll
+        for (int q = 0; q <= AR::kAccFloats; ++q) tot[q * NT] = 0.f;
+    }
     // cp.async walker over this thread's sequence: rows, chunks in reverse, steps forward
     const XT *const xbase = xrow;
     int wr = 0, wc = nc - 1, wt = 0;
@@ -1530,11 +1609,20 @@ dendsn_backward_kernel(const BwdArgs A) {
                 if (has_gv) gvp -= BN;
             }
         }
+        if (use_tot) {
+            AR::template acc_flush<NT>(acc, tot);
+            tot[AR::kAccFloats * NT] = __fadd_rn(tot[AR::kAccFloats * NT], gbeta);
+            gbeta = 0.f;
+        }
         xrow += rX;
         gsrow += jstep;
         gxrow += rX;
         if (has_gv) gvrow += jstep;
         j += jstep;
+    }
+    if (use_tot) {
+        AR::template acc_load<NT>(acc, tot);
+        gbeta = tot[AR::kAccFloats * NT];
     }
 
     // ---- parameter-gradient partials: per channel, fixed summation order
@@ -1683,7 +1771,7 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
 #pragma unroll
             for (int tt = L - 1; tt >= 0; --tt) {
                 const float2 vdp = tt > 0 ? hist[((tt > 0 ? tt - 1 : 0) * N2 + m) * NT] : f2(0.f);
-                hist[(tt * N2 + m) * NT] = AR::pair_back(lp, m, vdt, vdp, f2(dz[tt]), f2(0.f), Ad, acc);
+                hist[(tt * N2 + m) * NT] = AR::pair_back(lp, m, vdt, vdp, f2(-dz[tt]), f2(0.f), Ad, acc);
                 vdt = vdp;
             }
         }
@@ -1767,8 +1855,9 @@ dendsn_backward_rowpair_kernel(const BwdArgs A) {
     const int nrows = pos.nrows;
     const int nq = (nrows + 1) / 2;              // row pairs
 
-    // dynamic shared memory: history [L][KT][NT] float2, x [2][L][NT], dL/dS [2][L][NT],
-    // mask bytes [2][NT]; or (at the end) the reduction
+    // dynamic shared memory: history [L][KT][NT] float2, x [2][L][NT], dL/dS [2][2][L][NT]
+    // and mask bytes [2][2][NT] (two row pairs: the current one and the next); or (at the
+    // end) the reduction
     extern __shared__ float4 smem_f4[];
     char *const sregion = reinterpret_cast<char *>(smem_f4);
     float2 *const hist = reinterpret_cast<float2 *>(sregion) + threadIdx.x;
@@ -1777,7 +1866,7 @@ dendsn_backward_rowpair_kernel(const BwdArgs A) {
                                                    sizeof(XRaw) * 2 * L * NT) + threadIdx.x;
     uint32_t *const mring = reinterpret_cast<uint32_t *>(sregion + sizeof(float2) * L * KT * NT +
                                                          sizeof(XRaw) * 2 * L * NT +
-                                                         sizeof(float) * 2 * L * NT) + threadIdx.x;
+                                                         sizeof(float) * 4 * L * NT) + threadIdx.x;
     // neuron (within a sample) of the first row of the pair being fetched, for the masks
     const int nstep = (int)(jstep % g.N);
     int nf = (int)(j0 % g.N);
@@ -1794,22 +1883,25 @@ dendsn_backward_rowpair_kernel(const BwdArgs A) {
         }
         cp_async_commit();
     };
+    // dL/dS and mask bytes of row pair q into buffer q & 1, one row pair ahead of their use
     auto fetch_gs = [&](int q, float dep) {
         const int k = 2 * q;
+        float *const gbuf = gring + (q & 1) * 2 * L * NT;
+        uint32_t *const mbuf = mring + (q & 1) * 2 * NT;
         if (k < nrows) {
             const bool two = k + 1 < nrows;
             const float *p1 = gs0 + (int64_t)k * jstep;
 #pragma unroll
             for (int tt = 0; tt < L; ++tt) {
-                cp_async<4>(gring + tt * NT, p1 + (int64_t)tt * BN, dep);
-                if (two) cp_async<4>(gring + (L + tt) * NT, p1 + jstep + (int64_t)tt * BN, dep);
-                else gring[(L + tt) * NT] = 0.f;
+                cp_async<4>(gbuf + tt * NT, p1 + (int64_t)tt * BN, dep);
+                if (two) cp_async<4>(gbuf + (L + tt) * NT, p1 + jstep + (int64_t)tt * BN, dep);
+                else gbuf[(L + tt) * NT] = 0.f;
             }
             if (P.mask_mode == 2) {
                 int n2 = nf + nstep;
                 if (n2 >= g.N) n2 -= g.N;
-                cp_async<4>(mring, P.mask + (int64_t)nf * g.Kb + pos.sub * KT, dep);
-                cp_async<4>(mring + NT, P.mask + (int64_t)(two ? n2 : nf) * g.Kb + pos.sub * KT, dep);
+                cp_async<4>(mbuf, P.mask + (int64_t)nf * g.Kb + pos.sub * KT, dep);
+                cp_async<4>(mbuf + NT, P.mask + (int64_t)(two ? n2 : nf) * g.Kb + pos.sub * KT, dep);
                 nf = n2 + nstep;
                 if (nf >= g.N) nf -= g.N;
             }
@@ -1818,19 +1910,25 @@ dendsn_backward_rowpair_kernel(const BwdArgs A) {
     };
     fetch_x(0, 0.f);
     fetch_gs(0, 0.f);
+    float gdep = 0.f;   // a value computed from the last reads of the buffer fetch_gs refills
 
-    float2 ga[KT], ngxi[KT], ngz[KT], gk[KT];
+    float2 ga[KT], ngxi[KT], ngz[KT], ngk[KT];
 #pragma unroll
-    for (int c = 0; c < KT; ++c) { ga[c] = f2(0.f); ngxi[c] = f2(0.f); ngz[c] = f2(0.f); gk[c] = f2(0.f); }
+    for (int c = 0; c < KT; ++c) { ga[c] = f2(0.f); ngxi[c] = f2(0.f); ngz[c] = f2(0.f); ngk[c] = f2(0.f); }
     float2 gb = f2(0.f);
     for (int q = 0; q < nq; ++q) {
         const int k = 2 * q;
         const bool two = k + 1 < nrows;
         cp_async_wait<0>();
+        const float *const gcur = gring + (q & 1) * 2 * L * NT;
+        const uint32_t *const mcur = mring + (q & 1) * 2 * NT;
+        // the next pair's dL/dS and mask bytes go to the other buffer, read by the previous
+        // pair (gdep depends on those reads)
+        fetch_gs(q + 1, gdep);
         // the two rows' kappa * m and mask terms (exponent 0 / -inf, or m for the identity)
         float2 km2[KT], lm2[KT];
         if (P.mask_mode == 2) {
-            const uint32_t m1 = mring[0], m2 = mring[NT];
+            const uint32_t m1 = mcur[0], m2 = mcur[NT];
 #pragma unroll
             for (int c = 0; c < KT; ++c) {
                 const bool on1 = ((m1 >> (8 * c)) & 0xffu) != 0u, on2 = ((m2 >> (8 * c)) & 0xffu) != 0u;
@@ -1885,8 +1983,9 @@ dendsn_backward_rowpair_kernel(const BwdArgs A) {
         }
         fetch_x(q + 1, __fadd_rn(z[L - 1].x, z[L - 1].y));
 
-        // phase 2: the somas forward, then dL/dV^s backwards in time (dL/dZ = dL/dV^s)
-        float2 dz[L];
+        // phase 2: the somas forward, then dL/dV^s backwards in time (dL/dZ = dL/dV^s); ndz
+        // keeps -dL/dZ
+        float2 ndz[L];
         {
             float v1 = 0.f, v2 = 0.f;
             bool s1 = false, s2 = false;
@@ -1911,7 +2010,7 @@ dendsn_backward_rowpair_kernel(const BwdArgs A) {
                 }
                 const float2 dvds = ffma2(f2(kv), vs, f2(cs));
                 const float2 dvdv = make_float2(st1 ? b_spike : P.beta, st2 ? b_spike : P.beta);
-                const float2 ds = ffma2(dvds, dvn, make_float2(gring[tt * NT], gring[(L + tt) * NT]));
+                const float2 ds = ffma2(dvds, dvn, make_float2(gcur[tt * NT], gcur[(L + tt) * NT]));
                 const float2 xd = make_float2(__fsub_rn(vs.x, P.theta), __fsub_rn(vs.y, P.theta));
                 const float2 qd = ffma2(fmul2(f2(pi2), xd), xd, f2(1.f));
                 const float2 sg = make_float2(fast_rcp(qd.x), fast_rcp(qd.y));
@@ -1920,11 +2019,11 @@ dendsn_backward_rowpair_kernel(const BwdArgs A) {
                     const float *gp = A.gv + j0 + (int64_t)k * jstep + (int64_t)tt * BN;
                     dv = make_float2(__fadd_rn(dv.x, __ldcs(gp)), __fadd_rn(dv.y, two ? __ldcs(gp + jstep) : 0.f));
                 }
-                dz[tt] = dv;
+                ndz[tt] = neg2(dv);
                 dvn = dv;
             }
         }
-        fetch_gs(q + 1, __fadd_rn(dz[0].x, dz[0].y));
+        gdep = __fadd_rn(ndz[0].x, ndz[0].y);
 
         // phase 3: the dendritic reverse scan, one compartment at a time
 #pragma unroll
@@ -1935,23 +2034,23 @@ dendsn_backward_rowpair_kernel(const BwdArgs A) {
             for (int tt = L - 1; tt >= 0; --tt) {
                 const float2 vdp = tt > 0 ? hist[((tt > 0 ? tt - 1 : 0) * KT + c) * NT] : f2(0.f);
                 const float2 u = ffma2(vdt, f2(iz[c]), f2(nxi[c]));
-                const float2 gy = fmul2(km2[c], dz[tt]);
+                const float2 ngy = fmul2(km2[c], ndz[tt]);          // -dL/dY
                 float2 y, du;
                 if constexpr (PSI == PSI_MEXHAT) {
                     const float2 ss = fmul2(u, u);
                     const float2 t = ffma2(f2(kNegHalfLog2e), ss, lm2[c]);
                     const float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
                     y = ffma2(neg2(ss), e, e);
-                    const float2 w = fmul2(fadd2(ss, f2(-3.f)), e);
-                    du = fmul2(fmul2(w, u), gy);
+                    const float2 nw = ffma2(f2(2.f), e, y);        // -psi'(r) / r
+                    du = fmul2(nw, fmul2(u, ngy));
                 } else {
                     y = fmul2(lm2[c], make_float2(fabsf(u.x), fabsf(u.y)));
-                    du = make_float2(u.x > 0.f ? gy.x : (u.x < 0.f ? -gy.x : 0.f),
-                                     u.y > 0.f ? gy.y : (u.y < 0.f ? -gy.y : 0.f));
+                    du = make_float2(u.x > 0.f ? -ngy.x : (u.x < 0.f ? ngy.x : 0.f),
+                                     u.y > 0.f ? -ngy.y : (u.y < 0.f ? ngy.y : 0.f));
                 }
                 ngxi[c] = fadd2(ngxi[c], du);
                 ngz[c] = ffma2(u, du, ngz[c]);
-                gk[c] = ffma2(y, dz[tt], gk[c]);
+                ngk[c] = ffma2(y, ndz[tt], ngk[c]);
                 Ad = ffma2(f2(a[c]), Ad, du);
                 ga[c] = ffma2(Ad, vdp, ga[c]);
                 hist[(tt * KT + c) * NT] = ffma2(Ad, f2(iz[c]), f2(0.f));
@@ -1985,7 +2084,7 @@ dendsn_backward_rowpair_kernel(const BwdArgs A) {
         v[c] = __fmul_rn(__fadd_rn(ga[c].x, ga[c].y), iz[c]);
         v[KT + c] = -__fmul_rn(__fadd_rn(ngxi[c].x, ngxi[c].y), iz[c]);
         v[2 * KT + c] = -__fmul_rn(__fadd_rn(ngz[c].x, ngz[c].y), iz[c]);
-        v[3 * KT + c] = __fadd_rn(gk[c].x, gk[c].y);
+        v[3 * KT + c] = -__fadd_rn(ngk[c].x, ngk[c].y);
     }
     v[NA] = (BETA && pos.sub == 0) ? __fadd_rn(gb.x, gb.y) : 0.f;
 #pragma unroll
@@ -2003,8 +2102,24 @@ cudaError_t allow_smem(Kern kernel, size_t bytes) {
     return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
 }
 
+// Blocks of `kernel` (threads, bytes of dynamic shared memory) that fit on one SM, cached
+// per (kernel, threads, bytes) on the current device.
+cudaError_t resident_blocks(const void *kernel, int threads, size_t bytes, int *out);
+
+// Launches `kernel` on `blocks` blocks, or with `resident` non-null only reports how many of
+// its blocks fit on one SM.
+template <typename Kern, typename Args>
+cudaError_t launch_or_query(Kern kernel, const Args &a, int blocks, int threads, size_t bytes,
+                            cudaStream_t s, int *resident) {
+    cudaError_t e = allow_smem(kernel, bytes);
+    if (e != cudaSuccess) return e;
+    if (resident) return resident_blocks(reinterpret_cast<const void *>(kernel), threads, bytes, resident);
+    kernel<<<blocks, threads, bytes, s>>>(a);
+    return cudaGetLastError();
+}
+
 template <int K, int G, int PSI, int XT, int LAYOUT>
-cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s) {
+cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s, int *resident) {
     using T = typename XType<XT>::type;
     constexpr int KT = lane_compartments(K);
     using XI = XIO<T, KT, LAYOUT>;
@@ -2015,38 +2130,32 @@ cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s) {
         if (a.g.inner % 32 == 0 && a.g.TXn % 32 == 0) {
             const size_t smem = (size_t)kFwdDepth * NT * K * sizeof(T) +
                                 kappa_smem_bytes(a.p.mask_mode, K / G, NT);
-            cudaError_t e = allow_smem(dendsn_forward_staged_kernel<K, G, PSI, T>, smem);
-            if (e != cudaSuccess) return e;
-            dendsn_forward_staged_kernel<K, G, PSI, T><<<blocks, NT, smem, s>>>(a);
-            return cudaGetLastError();
+            return launch_or_query(dendsn_forward_staged_kernel<K, G, PSI, T>, a, blocks, NT, smem,
+                                   s, resident);
         }
     }
     const size_t smem = ((DENDSN_FWD_ASYNC && XI::kAsync) ? raw * fwd_depth<T, typename XI::Raw>() * NT : 0) +
                         kappa_smem_bytes(a.p.mask_mode, KT / G, NT);
-    cudaError_t e = allow_smem(dendsn_forward_kernel<K, G, PSI, T, LAYOUT>, smem);
-    if (e != cudaSuccess) return e;
-    dendsn_forward_kernel<K, G, PSI, T, LAYOUT><<<blocks, NT, smem, s>>>(a);
-    return cudaGetLastError();
+    return launch_or_query(dendsn_forward_kernel<K, G, PSI, T, LAYOUT>, a, blocks, NT, smem, s,
+                           resident);
 }
 
 template <int K, int G, int PSI, int XT, int L, int LAYOUT>
-cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
+cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s, int *resident) {
     using T = typename XType<XT>::type;
     constexpr int KT = bwd_lane_compartments(K, G, XT, L);
     constexpr int NT = bwd_threads(KT);
-    const size_t red = sizeof(float) * (acc_count<KT, G>() + 1) * NT;
+    const size_t red = red_bytes(acc_count<KT, G>() + 1, NT);
     constexpr bool shist = (L > 4) || KT >= 8;
     const size_t hist = shist ? sizeof(float) * (KT + 1) * L * NT : 0;
     using XI = XIO<T, KT, LAYOUT>;
     constexpr size_t xraw = sizeof(typename XI::Raw);
     const size_t ring = (DENDSN_BWD_ASYNC && shist && XI::kAsync) ? xraw * kBwdDepth * NT : 0;
-    const size_t smem = (red > hist + ring ? red : hist + ring) +
+    const size_t totals = row_totals<K, G, T, L>() ? sizeof(float) * (acc_count<KT, G>() + 1) * NT : 0;
+    const size_t smem = (red > hist + ring + totals ? red : hist + ring + totals) +
                         kappa_smem_bytes(a.p.mask_mode, KT / G, NT);
     auto go_smem = [&](auto kernel, size_t bytes) {
-        cudaError_t e = allow_smem(kernel, bytes);
-        if (e != cudaSuccess) return e;
-        kernel<<<blocks, NT, bytes, s>>>(a);
-        return cudaGetLastError();
+        return launch_or_query(kernel, a, blocks, NT, bytes, s, resident);
     };
     auto go = [&](auto kernel) { return go_smem(kernel, smem); };
     // 4-step rows of 8-compartment float32 neurons on two lanes: two rows per thread
@@ -2054,7 +2163,7 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s) {
     if constexpr (kRowPair) {
         if (a.g.T == 4 && !a.p.residual) {
             const size_t rp = sizeof(float2) * L * KT * NT + xraw * 2 * L * NT +
-                              sizeof(float) * 2 * L * NT + sizeof(uint32_t) * 2 * NT;
+                              sizeof(float) * 4 * L * NT + sizeof(uint32_t) * 4 * NT;
             const size_t rsm = red > rp ? red : rp;
             return a.want_beta ? go_smem(dendsn_backward_rowpair_kernel<PSI, LAYOUT, true>, rsm)
                                : go_smem(dendsn_backward_rowpair_kernel<PSI, LAYOUT, false>, rsm);

@@ -82,11 +82,13 @@ struct FinArgs {
 };
 
 // XT: 0 = float, 1 = bfloat16. LAYOUT: 0 = compartments innermost, 1 = the paper's
-// (C_o, P, H, W) layer layout. Defined in the instantiation units.
+// (C_o, P, H, W) layer layout. Defined in the instantiation units. With `resident` non-null
+// nothing is launched: *resident receives how many blocks of the kernel this call would
+// launch fit on one SM (the planner sizes grids in whole waves of that many blocks per SM).
 template <int K, int G, int PSI, int XT, int LAYOUT>
-cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s);
+cudaError_t launch_forward(const FwdArgs &a, int blocks, cudaStream_t s, int *resident);
 template <int K, int G, int PSI, int XT, int L, int LAYOUT>
-cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s);
+cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s, int *resident);
 cudaError_t launch_finalize(const FinArgs &a, cudaStream_t s);
 
 // Time-parallel kernels (tp_kernels.cu): one warp per neuron, for layers with at least

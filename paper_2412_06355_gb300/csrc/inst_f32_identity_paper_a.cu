@@ -5,8 +5,8 @@
 
 namespace dendsn {
 #define DENDSN_INST(K, G) \
-    template cudaError_t launch_forward<K, G, 0, 0, 1>(const FwdArgs &, int, cudaStream_t);     \
-    template cudaError_t launch_backward<K, G, 0, 0, 4, 1>(const BwdArgs &, int, cudaStream_t);
+    template cudaError_t launch_forward<K, G, 0, 0, 1>(const FwdArgs &, int, cudaStream_t, int *);     \
+    template cudaError_t launch_backward<K, G, 0, 0, 4, 1>(const BwdArgs &, int, cudaStream_t, int *);
 DENDSN_KG_LIST(DENDSN_INST)
 #undef DENDSN_INST
 }  // namespace dendsn

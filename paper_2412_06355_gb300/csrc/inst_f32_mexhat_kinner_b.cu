@@ -5,7 +5,7 @@
 
 namespace dendsn {
 #define DENDSN_INST(K, G) \
-    template cudaError_t launch_backward<K, G, 1, 0, 8, 0>(const BwdArgs &, int, cudaStream_t);
+    template cudaError_t launch_backward<K, G, 1, 0, 8, 0>(const BwdArgs &, int, cudaStream_t, int *);
 DENDSN_KG_LIST(DENDSN_INST)
 #undef DENDSN_INST
 }  // namespace dendsn
