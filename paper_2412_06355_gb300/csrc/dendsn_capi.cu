@@ -28,8 +28,19 @@ __global__ void param_grad_finalize_kernel(const FinArgs F) {
         const int ct_hi = (int)((((int64_t)c + 1) * g.inner - 1) / g.TXn);
         for (int ct = ct_lo; ct <= ct_hi; ++ct) {
             const int lc = c - (int)(((int64_t)ct * g.TXn) / g.inner);
-            for (int rg = 0; rg < g.nRG; ++rg)
-                sum = __fadd_rn(sum, F.partials[(((int64_t)rg * g.nCT + ct) * g.nch_max + lc) * NP + q]);
+            const float *p = F.partials + ((int64_t)ct * g.nch_max + lc) * NP + q;
+            const int64_t stride = (int64_t)g.nCT * g.nch_max * NP;   // between row groups
+            // unrolled so that the loads of eight row groups are in flight together; the
+            // additions keep their fixed order
+            int rg = 0;
+            for (; rg + 8 <= g.nRG; rg += 8) {
+                float v[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) v[u] = p[(int64_t)(rg + u) * stride];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) sum = __fadd_rn(sum, v[u]);
+            }
+            for (; rg < g.nRG; ++rg) sum = __fadd_rn(sum, p[(int64_t)rg * stride]);
         }
     }
     if (q < g.K) F.g_alpha[(int64_t)c * g.K + q] = F.stateless ? 0.f : sum;

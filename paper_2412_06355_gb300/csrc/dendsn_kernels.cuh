@@ -1656,8 +1656,14 @@ dendsn_backward_kernel(const BwdArgs A) {
 //   4. gather each step's dL/dX from shared memory and store it as one vector.
 // Every accumulator sees its terms in the same order as in dendsn_backward_kernel, so
 // the two kernels give bit-identical results.
+// Resident blocks of the phased backward: 3 (168 registers). 4 blocks at a 128-register cap
+// measured 3% slower on the deeper conv layer (552.6 -> 569.5 us; 4 bytes of spill, and the
+// compiler gives up instruction-level parallelism for the extra warps).
+#ifndef DENDSN_PHASED_MINB
+#define DENDSN_PHASED_MINB 3
+#endif
 template <int K, int PSI, typename XT, int L, bool BETA>
-__global__ void __launch_bounds__(bwd_threads(K), bwd_threads(K) == 128 ? 3 : 2)
+__global__ void __launch_bounds__(bwd_threads(K), bwd_threads(K) == 128 ? DENDSN_PHASED_MINB : 2)
 dendsn_backward_phased_kernel(const BwdArgs A) {
     constexpr int KT = K;
     constexpr int NT = bwd_threads(KT);
