@@ -1711,11 +1711,15 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
     float gbeta = 0.f;
     MaskAhead<AR, NT> mask;
     mask.init(P, g, j0, jstep, pos.chan, 0, pos.nrows, smem_f4);
-    for (int i = 0; i < pos.nrows; ++i) {
-        mask.advance(P, g, 0, i + 1 < pos.nrows, lp);
-        typename S1::Raw gsr[L];                 // grad_spikes of the row, used in phase 2
+    // grad_spikes of the row, used in phase 2; the next row's are requested right after it,
+    // so that phases 3 and 4 and the next recompute cover their latency
+    typename S1::Raw gsr[L];
+    if (pos.nrows > 0) {
 #pragma unroll
         for (int tt = 0; tt < L; ++tt) gsr[tt] = S1::load(gsrow + (int64_t)tt * BN);
+    }
+    for (int i = 0; i < pos.nrows; ++i) {
+        mask.advance(P, g, 0, i + 1 < pos.nrows, lp);
 
         // phase 1: recompute
         cp_async_wait<0>();
@@ -1767,6 +1771,10 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
                 dz[tt] = dv;
                 dvn = dv;
             }
+        }
+        if (i + 1 < pos.nrows) {
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) gsr[tt] = S1::load(gsrow + jstep + (int64_t)tt * BN);
         }
 
         // phase 3: the dendritic reverse scan, one pair at a time
