@@ -571,81 +571,67 @@ def time_layer(layer, args, world, dev):
 def time_e2e(layer, args, world, dev):
     """End to end through the C ABI from pinned host buffers, copies inside the timed region.
 
-    The batch is held on the host as `nch` contiguous sub-batches (samples are independent);
-    each sub-batch's H2D copy, forward + backward (C ABI, own stream) and D2H copy run on
-    three streams ordered by events, so both copy directions overlap each other and the
-    kernels. Every sub-batch call has the whole layer's columns, B / nch samples. Each
-    step's parameter gradients come back per sub-batch and are summed on the host while the
-    next step runs; the last step's sum is done before the clock stops. Timed on the wall
-    clock (host work included)."""
+    Each step is the headline call itself (one forward and one backward over the whole
+    batch) between a host->device copy of its inputs (x, dL/dS) and a device->host copy of
+    its results (spikes, dL/dX, the parameter gradients). Two sets of device buffers
+    alternate between steps, and the copies of each direction and the kernels run on three
+    streams ordered by events, so the next step's upload overlaps this step's download. The
+    host waits for each step's results before it enqueues the step after next. Timed on the
+    wall clock."""
     import torch
     import torch.distributed as dist
     from paper_2412_06355_gb300 import binding, distributed
-    w, x, gs = layer.w, layer.x, layer.gs
+    w, x, gs, cfg = layer.w, layer.x, layer.gs, layer.cfg
     alpha, xi, zeta, kappa = layer.prm
     mask = layer.mask
-    nch = next(c for c in (8, 4, 2, 1) if w.B % c == 0)
-    bc = w.B // nch
-    wc = layer.w_rank.with_(B=bc)
-    cfg_c = binding.config_of(wc)
     pin = dict(pin_memory=True)
-    x_h = [torch.empty((w.T, bc) + tuple(x.shape[2:]), dtype=x.dtype, **pin) for _ in range(nch)]
-    gs_h = [torch.empty((w.T, bc, w.N), dtype=gs.dtype, **pin) for _ in range(nch)]
-    for c in range(nch):
-        x_h[c].copy_(x[:, c * bc:(c + 1) * bc])
-        gs_h[c].copy_(gs[:, c * bc:(c + 1) * bc])
-    x_d = [torch.empty_like(t, device=dev) for t in x_h]
-    gs_d = [torch.empty_like(t, device=dev) for t in gs_h]
-    s_d = [torch.empty((w.T, bc, w.N), dtype=x.dtype, device=dev) for _ in range(nch)]
-    gx_d = [torch.empty_like(t) for t in x_d]
-    ws_c = [binding.workspace(cfg_c, dev) for _ in range(nch)]
+    x_h = torch.empty(x.shape, dtype=x.dtype, **pin)
+    gs_h = torch.empty(gs.shape, dtype=gs.dtype, **pin)
+    x_h.copy_(x)
+    gs_h.copy_(gs)
+    s_h = torch.empty((w.T, w.B, w.N), dtype=x.dtype, **pin)
+    gx_h = torch.empty(x.shape, dtype=x.dtype, **pin)
     ng = layer.grads.numel()
-    g_d = torch.empty((nch, ng), dtype=torch.float32, device=dev)
-    g_v = [distributed.split_param_grads(g_d[c], w.C, w.K, w.Kb) for c in range(nch)]
-    s_h = [torch.empty(t.shape, dtype=t.dtype, **pin) for t in s_d]
-    gx_h = [torch.empty(t.shape, dtype=t.dtype, **pin) for t in gx_d]
-    g_h = [torch.empty((nch, ng), dtype=torch.float32, **pin) for _ in range(2)]
-    h2d = sum(t.numel() * t.element_size() for t in x_h + gs_h)
-    d2h = (sum(t.numel() * t.element_size() for t in s_h + gx_h) +
-           g_h[0].numel() * g_h[0].element_size())
+    g_h = torch.empty(ng, dtype=torch.float32, **pin)
+    sets = []
+    for _ in range(2):
+        g_d = torch.empty(ng, dtype=torch.float32, device=dev)
+        sets.append(dict(x=torch.empty_like(x), gs=torch.empty_like(gs),
+                         s=torch.empty((w.T, w.B, w.N), dtype=x.dtype, device=dev),
+                         gx=torch.empty_like(x), ws=binding.workspace(cfg, dev), g=g_d,
+                         gv=distributed.split_param_grads(g_d, w.C, w.K, w.Kb)))
+    h2d = x_h.numel() * x_h.element_size() + gs_h.numel() * gs_h.element_size()
+    d2h = (s_h.numel() * s_h.element_size() + gx_h.numel() * gx_h.element_size() +
+           g_h.numel() * g_h.element_size())
     up, comp, down = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
     ev = lambda: torch.cuda.Event()                   # noqa: E731
-    loaded, computed, returned = ([ev() for _ in range(nch)] for _ in range(3))
-    all_done, grads_home = ev(), [ev(), ev()]
-    sums = []
+    loaded, computed, returned = ([ev(), ev()] for _ in range(3))
 
     def e2e_step(k):
-        for c in range(nch):
-            with torch.cuda.stream(up):
-                up.wait_event(computed[c])           # the previous step has read x_d[c]
-                x_d[c].copy_(x_h[c], non_blocking=True)
-                gs_d[c].copy_(gs_h[c], non_blocking=True)
-                loaded[c].record(up)
-            comp.wait_event(loaded[c])
-            comp.wait_event(returned[c])             # the previous step's D2H is done
-            saved_c, scratch_c = ws_c[c]
-            binding.dendsn_forward(cfg_c, x_d[c], alpha, xi, zeta, kappa, mask, s_d[c], None,
-                                   saved_c, comp)
-            binding.dendsn_backward(cfg_c, x_d[c], alpha, xi, zeta, kappa, mask, gs_d[c], None,
-                                    saved_c, gx_d[c], *g_v[c], scratch_c, comp)
-            computed[c].record(comp)
-            with torch.cuda.stream(down):
-                down.wait_event(computed[c])
-                s_h[c].copy_(s_d[c], non_blocking=True)
-                gx_h[c].copy_(gx_d[c], non_blocking=True)
-                returned[c].record(down)
+        i = k % 2
+        d = sets[i]
+        saved, scratch = d["ws"]
+        with torch.cuda.stream(up):
+            up.wait_event(computed[i])               # the step before last has read set i
+            d["x"].copy_(x_h, non_blocking=True)
+            d["gs"].copy_(gs_h, non_blocking=True)
+            loaded[i].record(up)
+        comp.wait_event(loaded[i])
+        comp.wait_event(returned[i])                 # set i's results of two steps ago are home
+        binding.dendsn_forward(cfg, d["x"], alpha, xi, zeta, kappa, mask, d["s"], None, saved,
+                               comp)
+        binding.dendsn_backward(cfg, d["x"], alpha, xi, zeta, kappa, mask, d["gs"], None, saved,
+                                d["gx"], *d["gv"], scratch, comp)
         if world > 1:
             with torch.cuda.stream(comp):
-                dist.all_reduce(g_d)                 # sums every sub-batch's row over ranks
-        all_done.record(comp)
+                dist.all_reduce(d["g"])              # the data-parallel gradient sum
+        computed[i].record(comp)
         with torch.cuda.stream(down):
-            down.wait_event(all_done)
-            g_h[k % 2].copy_(g_d, non_blocking=True)
-            grads_home[k % 2].record(down)
-
-    def host_sum(k):                                 # the step's parameter gradients
-        grads_home[k % 2].synchronize()
-        sums.append(g_h[k % 2].sum(dim=0))
+            down.wait_event(computed[i])
+            s_h.copy_(d["s"], non_blocking=True)
+            gx_h.copy_(d["gx"], non_blocking=True)
+            g_h.copy_(d["g"], non_blocking=True)
+            returned[i].record(down)
 
     ke = max(3, min(args.steps, 20))
     for k in range(3):
@@ -653,27 +639,24 @@ def time_e2e(layer, args, world, dev):
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    sums.clear()
     t0 = time.perf_counter()
     for k in range(ke):
         e2e_step(k)
         if k > 0:
-            host_sum(k - 1)
-    host_sum(ke - 1)
+            returned[(k - 1) % 2].synchronize()      # the previous step's results are on the host
     torch.cuda.synchronize()
     ems = (time.perf_counter() - t0) * 1e3
-    assert len(sums) == ke and all(bool(torch.isfinite(s).all()) for s in sums)
+    assert bool(torch.isfinite(g_h).all())
     if world > 1:
         t = torch.tensor([ems], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ems = float(t.item())
     return {"value": world * ke * w.neuron_steps / (ems / 1e3), "unit": UNIT,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": ke,
-            "ms_per_step": ems / ke, "sub_batches": nch, "sub_batch_B": bc, "streams": 3,
-            "timing": "wall clock; the per-sub-batch parameter gradients are summed on the "
-                      "host inside the timed region",
-            "launch_geometry": f"{nch} calls of B={bc} per step (the timed headline is one "
-                               f"call of B={w.B})"}
+            "ms_per_step": ems / ke, "streams": 3,
+            "timing": "wall clock, host waits for each step's results",
+            "launch_geometry": f"the headline call (one forward and one backward of B={w.B}), "
+                               "two device buffer sets alternating"}
 
 
 def layer_report(layer, timing, world, dev, peak, peak_kind, clock):
