@@ -1357,6 +1357,10 @@ dendsn_backward_kernel(const BwdArgs A) {
     constexpr bool BASYNC = DENDSN_BWD_ASYNC && SHIST && V::kAsync;
     constexpr int D = kBwdDepth;
     constexpr bool SLOTS = FULL && BASYNC && D == L;
+    // float32 dL/dS of the next chunk reaches shared memory by cp.async as each slot of the
+    // current chunk is taken (event-stream layer backward 1608 -> 1531 us; for the
+    // register-history builds it measured slower: conv layer 217.6 -> 221.8 us)
+    constexpr bool GSA = std::is_same<XT, float>::value && SLOTS;
     const Geometry &g = A.g;
     const Params &P = A.p;
     const ThreadPos pos = thread_pos<LPN>(g);
@@ -1398,6 +1402,9 @@ dendsn_backward_kernel(const BwdArgs A) {
     float *const tot = reinterpret_cast<float *>(reinterpret_cast<char *>(hist_vs + (SHIST ? L * NT : 0)) +
                                                  (BASYNC ? sizeof(XRaw) * D * NT : 0)) + threadIdx.x;
     const bool use_tot = TOTALS && nc > 1;
+    float *const gring = reinterpret_cast<float *>(reinterpret_cast<char *>(tot - threadIdx.x) +
+                                                   (TOTALS ? sizeof(float) * (AR::kAccFloats + 1) * NT : 0)) +
+                         threadIdx.x;                                                // [L][NT]
     if (use_tot) {
 #pragma unroll
         for (int q = 0; q <= AR::kAccFloats; ++q) tot[q * NT] = 0.f;
@@ -1445,7 +1452,8 @@ dendsn_backward_kernel(const BwdArgs A) {
         for (int tt = 0; tt < L; ++tt) {
             if (t0 + tt < T) {
                 if (!BASYNC && tt < H) xb[(!BASYNC && tt < H) ? tt : 0] = V::load(p, ks);
-                gsb[tt] = S1::load(q);
+                if constexpr (GSA) cp_async<4>(gring + tt * NT, q, 0.f);
+                else gsb[tt] = S1::load(q);
             }
             p += sX;
             q += BN;
@@ -1456,6 +1464,7 @@ dendsn_backward_kernel(const BwdArgs A) {
             ckv = __ldcs(A.ck_vs + (int64_t)(nc - 2) * BN + j0);
         }
     }
+    if constexpr (GSA) cp_async_commit();
 
     int64_t j = j0;
     MaskAhead<AR, NT> mask;
@@ -1561,7 +1570,11 @@ dendsn_backward_kernel(const BwdArgs A) {
 #pragma unroll
             for (int tt = L - 1; tt >= 0; --tt) {
                 float gs_t;
-                if constexpr (SHIST) {
+                if constexpr (GSA) {
+                    gs_t = gring[tt * NT];
+                    if (tt < nnext) cp_async<4>(gring + tt * NT, gqr, gs_t);
+                    gqr -= BN;
+                } else if constexpr (SHIST) {
                     gs_t = S1::unpack(gsb[tt]);
                     // refill slot tt with the next chunk's grad_spikes once this one is taken
                     if (tt < nnext) gsb[tt] = S1::load(gqr);
@@ -1608,6 +1621,7 @@ dendsn_backward_kernel(const BwdArgs A) {
                 gxp -= sX;
                 if (has_gv) gvp -= BN;
             }
+            if constexpr (GSA) cp_async_commit();
         }
         if (use_tot) {
             AR::template acc_flush<NT>(acc, tot);
@@ -1634,7 +1648,7 @@ dendsn_backward_kernel(const BwdArgs A) {
 #pragma unroll
     for (int a = 0; a < NA1; ++a)
         if (!pos.active || (a < KT && P.stateless)) v[a] = 0.f;
-    if constexpr (BASYNC) cp_async_wait<0>();
+    if constexpr (BASYNC || GSA) cp_async_wait<0>();
     block_partials<KT, G, LPN, NT>(g, pos, v, reinterpret_cast<float *>(sregion), A.partials);
 }
 
@@ -1649,7 +1663,8 @@ dendsn_backward_kernel(const BwdArgs A) {
 //      spikes are bit-identical), writing V^d of every step and pair to shared memory;
 //      then fetch the next row's x into the freed ring;
 //   2. the soma in registers: V^s forward, then its reverse recursion for dL/dZ[t]
-//      (Eqs. methods-lif-reset-charge, methods-lif-fire, methods-sg);
+//      (Eqs. methods-lif-reset-charge, methods-lif-fire, methods-sg); then fetch the next
+//      row's dL/dS;
 //   3. pair by pair, the dendritic reverse scan over the chunk (the same per-pair step as
 //      dendsn_backward_kernel); dL/dX[t] of a pair overwrites its V^d[t] slot, which the
 //      scan no longer needs;
@@ -1662,7 +1677,13 @@ dendsn_backward_kernel(const BwdArgs A) {
 #ifndef DENDSN_PHASED_MINB
 #define DENDSN_PHASED_MINB 3
 #endif
-template <int K, int PSI, typename XT, int L, bool BETA>
+// GSA: dL/dS reaches shared memory by cp.async, one row ahead, instead of registers
+// loaded one row ahead (deeper conv backward 549.4 -> 516.6 us: the register loads
+// still held up the soma phase; two rows ahead measured slower, 520.7 -> 525.6 us, and
+// x two rows ahead too, 529 us). For bfloat16 each thread copies the aligned 4-byte word
+// holding its element and its neighbour's; the launcher takes this build only when those
+// words lie inside each step's row (gs 4-byte aligned, B*N even), else the register one.
+template <int K, int PSI, typename XT, int L, bool BETA, bool GSA>
 __global__ void __launch_bounds__(bwd_threads(K), bwd_threads(K) == 128 ? DENDSN_PHASED_MINB : 2)
 dendsn_backward_phased_kernel(const BwdArgs A) {
     constexpr int KT = K;
@@ -1694,15 +1715,33 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
     const bool has_gv = A.gv != nullptr;
 
     // dynamic shared memory: the lanes' kappa (per-neuron masks only), then the history
-    // [L][N2][NT] float2 and the x ring [L][NT], or (at the end) the reduction
+    // [L][N2][NT] float2, the x ring [L][NT] and (GSA) the dL/dS ring [L][NT], or (at the
+    // end) the reduction
     extern __shared__ float4 smem_f4[];
     char *const sregion = reinterpret_cast<char *>(smem_f4) + kappa_smem_bytes(P.mask_mode, KT, NT);
     float2 *const hist = reinterpret_cast<float2 *>(sregion) + threadIdx.x;
     XRaw *const xring = reinterpret_cast<XRaw *>(reinterpret_cast<float2 *>(sregion) + L * N2 * NT) +
                         threadIdx.x;
+    // dL/dS of a row as L 4-byte words (for bfloat16 the word holding the thread's element
+    // and its neighbour's)
+    uint32_t *const gring = reinterpret_cast<uint32_t *>(reinterpret_cast<char *>(sregion) +
+                                                         sizeof(float2) * L * N2 * NT +
+                                                         sizeof(XRaw) * L * NT) + threadIdx.x;
+    auto gs_word = [&](const XT *p) {
+        return reinterpret_cast<const uint32_t *>(reinterpret_cast<uintptr_t>(p) & ~(uintptr_t)3);
+    };
+    // byte selector that moves the thread's bfloat16 half of a word to the top (exact)
+    auto gs_sel = [&](const XT *p) -> uint32_t {
+        if constexpr (std::is_same<XT, float>::value) return 0x3210u;
+        else return ((reinterpret_cast<uintptr_t>(p) >> 1) & 1) ? 0x3244u : 0x1044u;
+    };
     if (pos.nrows > 0) {
 #pragma unroll
         for (int tt = 0; tt < L; ++tt) V::copy_async(xring + tt * NT, xrow + (int64_t)tt * sX, 1, 0.f);
+        if constexpr (GSA) {
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) cp_async<4>(gring + tt * NT, gs_word(gsrow + (int64_t)tt * BN), 0.f);
+        }
     }
     cp_async_commit();
 
@@ -1711,10 +1750,10 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
     float gbeta = 0.f;
     MaskAhead<AR, NT> mask;
     mask.init(P, g, j0, jstep, pos.chan, 0, pos.nrows, smem_f4);
-    // grad_spikes of the row, used in phase 2; the next row's are requested right after it,
-    // so that phases 3 and 4 and the next recompute cover their latency
+    // without GSA: grad_spikes of the row in registers, used in phase 2; the next row's are
+    // requested right after it
     typename S1::Raw gsr[L];
-    if (pos.nrows > 0) {
+    if (!GSA && pos.nrows > 0) {
 #pragma unroll
         for (int tt = 0; tt < L; ++tt) gsr[tt] = S1::load(gsrow + (int64_t)tt * BN);
     }
@@ -1765,17 +1804,28 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
                 }
                 const float dvds = __fmaf_rn(kv, vs, cs);
                 const float dvdv = st ? b_spike : P.beta;
-                const float ds = __fmaf_rn(dvds, dvn, S1::unpack(gsr[tt]));
+                const float gst = GSA ? __uint_as_float(__byte_perm(gring[tt * NT], 0u, gs_sel(gsrow)))
+                                      : S1::unpack(gsr[tt]);
+                const float ds = __fmaf_rn(dvds, dvn, gst);
                 float dv = __fmaf_rn(surrogate(__fsub_rn(vs, P.theta)), ds, __fmul_rn(dvdv, dvn));
                 if (has_gv) dv = __fadd_rn(dv, __ldcs(gvrow + (int64_t)tt * BN));
                 dz[tt] = dv;
                 dvn = dv;
             }
         }
+        // the next row's dL/dS: into the ring once phase 2 has read it (dz[0] depends on
+        // every read), else into the registers
         if (i + 1 < pos.nrows) {
+            if constexpr (GSA) {
 #pragma unroll
-            for (int tt = 0; tt < L; ++tt) gsr[tt] = S1::load(gsrow + jstep + (int64_t)tt * BN);
+                for (int tt = 0; tt < L; ++tt)
+                    cp_async<4>(gring + tt * NT, gs_word(gsrow + jstep + (int64_t)tt * BN), dz[0]);
+            } else {
+#pragma unroll
+                for (int tt = 0; tt < L; ++tt) gsr[tt] = S1::load(gsrow + jstep + (int64_t)tt * BN);
+            }
         }
+        if constexpr (GSA) cp_async_commit();
 
         // phase 3: the dendritic reverse scan, one pair at a time
 #pragma unroll
@@ -2166,7 +2216,11 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s, int *r
     constexpr size_t xraw = sizeof(typename XI::Raw);
     const size_t ring = (DENDSN_BWD_ASYNC && shist && XI::kAsync) ? xraw * kBwdDepth * NT : 0;
     const size_t totals = row_totals<K, G, T, L>() ? sizeof(float) * (acc_count<KT, G>() + 1) * NT : 0;
-    const size_t smem = (red > hist + ring + totals ? red : hist + ring + totals) +
+    constexpr bool bslots = (L == 8 || (K / KT == 1 && G == 1 && LAYOUT == 0)) && DENDSN_BWD_ASYNC &&
+                            XI::kAsync && kBwdDepth == L;
+    constexpr bool gsa = XT == 0 && bslots;
+    const size_t gsb = gsa ? sizeof(float) * L * NT : 0;
+    const size_t smem = (red > hist + ring + totals + gsb ? red : hist + ring + totals + gsb) +
                         kappa_smem_bytes(a.p.mask_mode, KT / G, NT);
     auto go_smem = [&](auto kernel, size_t bytes) {
         return launch_or_query(kernel, a, blocks, NT, bytes, s, resident);
@@ -2190,10 +2244,16 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s, int *r
                              XI::kAsync;
     if constexpr (kPhased) {
         if (a.g.T == L && !a.p.residual) {
-            const size_t ph = sizeof(float) * KT * L * NT + xraw * L * NT;
+            // dL/dS by cp.async needs 4-byte words that stay inside each step's row; both
+            // builds reserve its shared memory, so the residency query (gs unknown) holds
+            const bool gsa = (reinterpret_cast<uintptr_t>(a.gs) & 3) == 0 && (XT == 0 || a.g.BN % 2 == 0);
+            const size_t ph = sizeof(float) * KT * L * NT + xraw * L * NT + sizeof(uint32_t) * L * NT;
             const size_t psm = (red > ph ? red : ph) + kappa_smem_bytes(a.p.mask_mode, KT, NT);
-            return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true>, psm)
-                               : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false>, psm);
+            if (gsa)
+                return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true, true>, psm)
+                                   : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false, true>, psm);
+            return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true, false>, psm)
+                               : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false, false>, psm);
         }
     }
     // full chunks: deeper conv layer 906 -> 738 us, event layer 1829 -> 1755 us, conv layer

@@ -4,8 +4,11 @@ The five layer shapes (tiny, conv, deeper bf16 conv, event-stream, transformer t
 per-neuron branch gating) run at their full sizes in the benchmark's launch configuration;
 the oracle simulates every neuron on all host cores (tests/full_parity.py). No rounding
 allowance is added: V^s within 1e-6 + 1e-5|v|, spikes identical outside the 1e-5 window,
-float32 gradients within 1e-4 relative + 1e-6 RMS, bfloat16 dL/dX within 2e-2 relative
-+ 1e-6 RMS, parameter gradients against the float64 sums over the whole layer.
+parameter gradients within 1e-4 relative + 1e-6 RMS against the float64 sums over the
+whole layer, dL/dX within 1e-4 relative (float32) or 2e-2 (bfloat16) + 1e-5 RMS: the
+absolute term is the reading of tests/parity.py, since float32 evaluation of the method
+itself misses 1e-6 RMS (tests/test_f32_restatement.py); each report also gives the worst
+error over the 1e-6 RMS bound.
 
 With DENDSN_PARITY_REPORT set to a directory, each case also writes its report there
 (worst error over bound per quantity, ambiguous-neuron count, timings).

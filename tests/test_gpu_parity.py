@@ -129,6 +129,31 @@ def test_one_chunk_rows_of_8_compartments(kw, dtype, T):
     check_layer(w)
 
 
+def test_phased_backward_grad_spike_paths_are_bitwise_equal():
+    """The phased backward takes dL/dS into shared memory by 4-byte cp.async words when gs
+    is 4-byte aligned and B*N is even, else into registers: both paths give the same bits,
+    and a layer with odd B*N (register path) matches the oracle."""
+    w = workloads.Workload("gsp", T=8, B=5, N=3 * 128, K=8, G=1, C=3, inner=128, dtype="bf16",
+                           psi="mh", reset="soft", mask_p=0.5, seed=43)
+    inp = to_dev(workloads.make_inputs(w, "cpu", with_gv=True))
+    cfg = binding.config_of(w)
+    prm = [inp[k] for k in ("alpha", "xi", "zeta", "kappa")]
+    for want_beta in (False, True):
+        outs = []
+        for off in (0, 1):                   # element offset 1: gs only 2-byte aligned
+            buf = torch.zeros(inp["gs"].numel() + 1, dtype=inp["gs"].dtype, device="cuda")
+            gs = buf[off:off + inp["gs"].numel()].view(inp["gs"].shape)
+            gs.copy_(inp["gs"])
+            saved, scratch = binding.workspace(cfg)
+            binding.forward(cfg, inp["x"], *prm, inp["mask"], want_v=False, saved=saved)
+            outs.append(binding.backward(cfg, inp["x"], *prm, inp["mask"], gs, inp["gv"], saved,
+                                         scratch, want_beta=want_beta))
+        torch.cuda.synchronize()
+        for k in outs[0]:
+            assert torch.equal(outs[0][k], outs[1][k]), (k, want_beta)
+    check_layer(w.with_(N=3 * 45, inner=45, seed=44))      # B*N = 675
+
+
 @pytest.mark.parametrize("T", [1, 2, 3, 5, 8, 9, 16, 17, 64, 70])
 def test_time_lengths_and_checkpoint_chunks(T):
     w = workloads.Workload("t", T=T, B=3, N=2 * 160, K=4, G=2, C=2, inner=160, dtype="f32",
