@@ -98,10 +98,15 @@ typedef struct {
 
 /*
  * Sizes of the two caller-owned device buffers a forward/backward pair needs.
- *   saved_bytes  : state checkpoints the forward writes and the backward reads
- *                  (recompute with checkpointing, Results "Constructing deep
- *                  DendSNNs"); 0 when T is short enough to recompute from X alone.
- *                  16-byte aligned. Must outlive the backward.
+ *   saved_bytes  : state the forward writes and the backward reads. For T > 8,
+ *                  checkpoints of (V^d, V^s) every 8 steps (recompute with
+ *                  checkpointing, Results "Constructing deep DendSNNs"). For layers
+ *                  whose backward serves each 8-compartment neuron on one thread over
+ *                  a single chunk (K = 8, G = 1, compartments innermost, no residual
+ *                  term, T = 8, or T = 4 with bfloat16 x), V^s [T, B, N] float32, so
+ *                  that the backward rescans only V^d; optional there (NULL in both
+ *                  calls: the backward recomputes V^s from x, with the same bits).
+ *                  Otherwise 0. 16-byte aligned. Must outlive the backward.
  *   scratch_bytes: per-block partial sums of the parameter gradients, used only by
  *                  dendsn_backward. 16-byte aligned. Contents need no initialisation.
  * Either output pointer may be NULL.
@@ -117,8 +122,8 @@ dendsn_status dendsn_workspace_size(const dendsn_config *cfg, size_t *saved_byte
  *   alpha..kappa, mask: parameters as above (read)
  *   spikes   [T,B,N] output (written)
  *   v_out    [T,B,N] float32 somatic potential V^s (written), or NULL
- *   saved    checkpoint buffer of saved_bytes (written), or NULL when no backward
- *            will follow; ignored when saved_bytes == 0
+ *   saved    buffer of saved_bytes (written), or NULL when no backward will follow;
+ *            ignored when saved_bytes == 0
  */
 dendsn_status dendsn_forward(const dendsn_config *cfg, const void *x, const float *alpha,
                              const float *xi, const float *zeta, const float *kappa,
@@ -129,7 +134,9 @@ dendsn_status dendsn_forward(const dendsn_config *cfg, const void *x, const floa
  * Fused reverse-time backward (BPTT with the arctan surrogate, Eq. methods-sg). The
  * forward of each checkpoint interval is recomputed from x in registers.
  *   grad_spikes [T,B,N] dL/dS (read); grad_v [T,B,N] float32 dL/dV^s (read) or NULL
- *   saved       the buffer the forward filled (read); may be NULL if saved_bytes == 0
+ *   saved       the buffer the forward of the same inputs filled (read); may be NULL
+ *               when T <= 8 if it was NULL in the forward too (a buffer the forward did
+ *               not fill gives wrong gradients, it is not detected)
  *   grad_x      [T,B,N,K] dL/dX (written)
  *   grad_alpha, grad_xi, grad_zeta, grad_kappa: parameter gradients summed over time,
  *               samples and the neurons of each channel (written, deterministic order).

@@ -115,6 +115,7 @@ struct Plan {
     Geometry gf, gb;   // forward and backward tilings (block sizes may differ)
     int blocks_f, blocks_b;
     size_t saved_bytes, scratch_bytes, ck_vd_bytes;
+    bool keep_vs;      // saved holds V^s [T][BN] for the single-chunk (phased) backward
     int sx;            // bytes per x element
     int layout;        // 0 compartments innermost, 1 the paper's layer layout
     bool tp;           // the time-parallel kernels (one warp per neuron)
@@ -308,10 +309,15 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl) {
         pl->gf.n_ck = pl->gb.n_ck = 0;                 // the backward recomputes from x alone
         pl->scratch_bytes = ((size_t)BN * NP * sizeof(float) + 15) / 16 * 16;
         pl->ck_vd_bytes = pl->saved_bytes = 0;
+        pl->keep_vs = false;
         return DENDSN_OK;
     }
     pl->ck_vd_bytes = (size_t)g.n_ck * (size_t)BN * c.K * sizeof(float);
     pl->saved_bytes = pl->ck_vd_bytes + (size_t)g.n_ck * (size_t)BN * sizeof(float);
+    // rows of one chunk of whole 8-compartment neurons (the phased backward): the forward
+    // keeps V^s, so that the backward recomputes only the compartment scan
+    pl->keep_vs = takes_phased_backward(c.K, c.G, KTB, pl->layout, c.T, g.L, c.residual != 0);
+    if (pl->keep_vs) pl->saved_bytes = (size_t)c.T * (size_t)BN * sizeof(float);
     pl->saved_bytes = (pl->saved_bytes + 15) / 16 * 16;
     return DENDSN_OK;
 }
@@ -445,6 +451,7 @@ dendsn_status dendsn_forward(const dendsn_config *cfg, const void *x, const floa
     a.ck_vd = (saved && pl.gf.n_ck > 0) ? static_cast<float *>(saved) : nullptr;
     a.ck_vs = a.ck_vd ? reinterpret_cast<float *>(static_cast<char *>(saved) + pl.ck_vd_bytes)
                       : nullptr;
+    a.vs_keep = (saved && pl.keep_vs) ? static_cast<float *>(saved) : nullptr;
     cudaError_t e = pl.tp ? dispatch_forward_tp(*cfg, pl.layout, a, static_cast<cudaStream_t>(stream))
                           : dispatch_forward(*cfg, pl.layout, a, pl.blocks_f, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess)
@@ -498,6 +505,7 @@ dendsn_status backward_impl(const dendsn_config *cfg, const void *x, const float
         a.ck_vs = pl.gb.n_ck > 0 ? reinterpret_cast<const float *>(
                                       static_cast<const char *>(saved) + pl.ck_vd_bytes)
                                 : nullptr;
+        a.vs_saved = (saved && pl.keep_vs) ? static_cast<const float *>(saved) : nullptr;
         a.gx = grad_x;
         a.partials = static_cast<float *>(scratch);
         a.want_beta = grad_beta != nullptr;

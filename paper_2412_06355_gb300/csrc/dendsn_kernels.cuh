@@ -943,6 +943,10 @@ dendsn_forward_kernel(const FwdArgs A) {
                                   lane_x_offset<LAYOUT>(j0, pos.sub, KT, K, g.inner);
     XT *__restrict__ srow = static_cast<XT *>(A.spikes) + j0;
     float *vrow = A.v_out ? A.v_out + j0 : nullptr;
+    // the kept V^s arises only for layers of the phased backward (one 8-compartment lane per
+    // neuron, compartments innermost); elsewhere krow is null at compile time
+    constexpr bool can_keep = K == 8 && G == 1 && LAYOUT == 0;
+    float *krow = (can_keep && A.vs_keep) ? A.vs_keep + j0 : nullptr;
     const bool write_ck = (A.ck_vd != nullptr) && g.n_ck > 0 && pos.active;
     const bool store = pos.active && pos.sub == 0;
     const bool residual = P.residual != 0;
@@ -971,12 +975,14 @@ dendsn_forward_kernel(const FwdArgs A) {
         // The step loop is specialised on whether V^s and checkpoints are written and on
         // whether T divides the ring depth (then the step fetched D steps ahead is the
         // same step D/T rows further on: no walker needed).
-        auto rows = [&](auto extra, auto div, auto tc) {
+        auto rows = [&](auto extra, auto div, auto tc, auto keep) {
             // EXTRA: V^s output and/or checkpoints requested (each still tested inside);
             // TC > 0: T == TC known at compile time (the step loop unrolls; slots are the
-            // row's first slot plus the step)
+            // row's first slot plus the step); KEEP: V^s kept for the backward (A.vs_keep
+            // non-null; a separate build, so that the other loops carry no test for it)
             constexpr bool EXTRA = decltype(extra)::value, DIV = decltype(div)::value;
             constexpr int TC = decltype(tc)::value;
+            constexpr bool KEEP = decltype(keep)::value;
             int slot = 0;
             int64_t j = j0;
             const int rows_ahead = DIV ? D / T : 0;
@@ -984,6 +990,7 @@ dendsn_forward_kernel(const FwdArgs A) {
             const XT *xr = xrow;
             XT *sr = srow;
             float *vr = vrow;
+            float *kr = KEEP ? krow : nullptr;
             MaskAhead<AR, NT> mask;
             mask.init(P, g, j0, jstep, pos.chan, pos.sub, pos.nrows, fwd_smem);
             for (int i = 0; i < pos.nrows; ++i) {
@@ -994,6 +1001,7 @@ dendsn_forward_kernel(const FwdArgs A) {
                 bool s = false;
                 XT *sp = sr;
                 float *vp = vr;
+                float *kp = kr;
                 const XT *cp = xr;                       // this step's x in global memory
                 const bool fetch_row = i + rows_ahead < pos.nrows;
                 auto step = [&](int t, int sl) {
@@ -1018,8 +1026,10 @@ dendsn_forward_kernel(const FwdArgs A) {
                         if constexpr (EXTRA) {
                             if (vp) __stcs(vp, v);
                         }
+                        if constexpr (KEEP) __stcs(kp, v);
                     }
                     sp += BN;
+                    if constexpr (KEEP) kp += BN;
                     if constexpr (EXTRA) {
                         if (vp) vp += BN;
                         if (write_ck && ((t + 1) & (g.L - 1)) == 0 && t + 1 < T) {
@@ -1046,21 +1056,44 @@ dendsn_forward_kernel(const FwdArgs A) {
                 if constexpr (EXTRA) {
                     if (vr) vr += jstep;
                 }
+                if constexpr (KEEP) kr += jstep;
                 j += jstep;
             }
         };
         using yes = std::true_type;
         using no = std::false_type;
         using tc0 = std::integral_constant<int, 0>;
+        using tc4 = std::integral_constant<int, 4>;
+        using tc8 = std::integral_constant<int, 8>;
         const bool div = (D % T) == 0;
-        if (vrow != nullptr || write_ck) {
-            if (div) rows(yes{}, yes{}, tc0{}); else rows(yes{}, no{}, tc0{});
+        const bool keep = can_keep && krow != nullptr;
+        if (vrow != nullptr || write_ck || (keep && !(div && (T == 4 || T == 8)))) {
+            if constexpr (can_keep) {
+                if (keep) {
+                    if (div) rows(yes{}, yes{}, tc0{}, yes{}); else rows(yes{}, no{}, tc0{}, yes{});
+                    cp_async_wait<0>();
+                    return;
+                }
+            }
+            if (div) rows(yes{}, yes{}, tc0{}, no{}); else rows(yes{}, no{}, tc0{}, no{});
         } else if (div) {
-            if (T == 4) rows(no{}, yes{}, std::integral_constant<int, 4>{});
-            else if (T == 8) rows(no{}, yes{}, std::integral_constant<int, 8>{});
-            else rows(no{}, yes{}, tc0{});
+            if (T == 4) {
+                if constexpr (can_keep) {
+                    if (keep) rows(no{}, yes{}, tc4{}, yes{}); else rows(no{}, yes{}, tc4{}, no{});
+                } else {
+                    rows(no{}, yes{}, tc4{}, no{});
+                }
+            } else if (T == 8) {
+                if constexpr (can_keep) {
+                    if (keep) rows(no{}, yes{}, tc8{}, yes{}); else rows(no{}, yes{}, tc8{}, no{});
+                } else {
+                    rows(no{}, yes{}, tc8{}, no{});
+                }
+            } else {
+                rows(no{}, yes{}, tc0{}, no{});
+            }
         } else {
-            rows(no{}, no{}, tc0{});
+            rows(no{}, no{}, tc0{}, no{});
         }
         cp_async_wait<0>();
         return;
@@ -1087,6 +1120,7 @@ dendsn_forward_kernel(const FwdArgs A) {
         bool s = false;
         XT *sp = srow;
         float *vp = vrow;
+        float *kp = krow;
         for (int c = 0; c < nb; ++c) {
             const int t0 = c * L;
             const int ncur = min(L, T - t0);                       // steps of this batch
@@ -1109,9 +1143,11 @@ dendsn_forward_kernel(const FwdArgs A) {
                     if (store) {
                         Scalar<XT>::store_spike(sp, s);
                         if (vp) __stcs(vp, v);
+                        if (kp) __stcs(kp, v);
                     }
                     sp += BN;
                     if (vp) vp += BN;
+                    if (kp) kp += BN;
                 }
             }
             if (write_ck && t0 + L < T && ((t0 + L) & (g.L - 1)) == 0) {
@@ -1125,6 +1161,7 @@ dendsn_forward_kernel(const FwdArgs A) {
         xrow += rX;
         srow += jstep;
         if (vrow) vrow += jstep;
+        if (krow) krow += jstep;
         j += jstep;
     }
 }
@@ -1683,7 +1720,11 @@ dendsn_backward_kernel(const BwdArgs A) {
 // x two rows ahead too, 529 us). For bfloat16 each thread copies the aligned 4-byte word
 // holding its element and its neighbour's; the launcher takes this build only when those
 // words lie inside each step's row (gs 4-byte aligned, B*N even), else the register one.
-template <int K, int PSI, typename XT, int L, bool BETA, bool GSA>
+// VS: V^s comes from the forward (A.vs_saved, by cp.async with dL/dS) instead of being
+// recomputed: phase 1 then only rescans V^d and phase 2 starts at the reverse recursion
+// (deeper conv backward 515.9 -> 461.8 us, for a forward that writes 4 more bytes per
+// neuron-step).
+template <int K, int PSI, typename XT, int L, bool BETA, bool GSA, bool VS>
 __global__ void __launch_bounds__(bwd_threads(K), bwd_threads(K) == 128 ? DENDSN_PHASED_MINB : 2)
 dendsn_backward_phased_kernel(const BwdArgs A) {
     constexpr int KT = K;
@@ -1695,6 +1736,7 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
     using AR = Arith<KT, 1, PSI, XT>;
     using XRaw = typename V::Raw;
     static_assert(KT % 2 == 0 && AR::KTb == KT, "paired engine only");
+    static_assert(!VS || GSA, "the kept V^s arrives with dL/dS");
     const Geometry &g = A.g;
     const Params &P = A.p;
     const ThreadPos pos = thread_pos<1>(g);
@@ -1727,6 +1769,9 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
     uint32_t *const gring = reinterpret_cast<uint32_t *>(reinterpret_cast<char *>(sregion) +
                                                          sizeof(float2) * L * N2 * NT +
                                                          sizeof(XRaw) * L * NT) + threadIdx.x;
+    // VS: the kept V^s of a row [L][NT] after the dL/dS ring
+    float *const vring = reinterpret_cast<float *>(gring + L * NT);
+    const float *vsrow = VS ? A.vs_saved + j0 : nullptr;
     auto gs_word = [&](const XT *p) {
         return reinterpret_cast<const uint32_t *>(reinterpret_cast<uintptr_t>(p) & ~(uintptr_t)3);
     };
@@ -1741,6 +1786,10 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
         if constexpr (GSA) {
 #pragma unroll
             for (int tt = 0; tt < L; ++tt) cp_async<4>(gring + tt * NT, gs_word(gsrow + (int64_t)tt * BN), 0.f);
+        }
+        if constexpr (VS) {
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) cp_async<4>(vring + tt * NT, vsrow + (int64_t)tt * BN, 0.f);
         }
     }
     cp_async_commit();
@@ -1762,7 +1811,8 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
 
         // phase 1: recompute
         cp_async_wait<0>();
-        float z[L];
+        float z[L];                              // Z, then V^s (VS: V^s from the start)
+        float xdep;                              // depends on every read of the x ring
         {
             typename AR::St vd;
             AR::zero(vd);
@@ -1770,28 +1820,38 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
             for (int tt = 0; tt < L; ++tt) {
                 float xv[KT];
                 V::unpack(xring[tt * NT], xv);
-                z[tt] = AR::step(lp, vd, xv, false, 0.f);
+                if constexpr (VS) {
+#pragma unroll
+                    for (int m = 0; m < N2; ++m)
+                        vd.v[m] = ffma2(lp.a[m], vd.v[m], make_float2(xv[2 * m], xv[2 * m + 1]));
+                    z[tt] = vring[tt * NT];
+                } else {
+                    z[tt] = AR::step(lp, vd, xv, false, 0.f);
+                }
 #pragma unroll
                 for (int m = 0; m < N2; ++m) hist[(tt * N2 + m) * NT] = vd.v[m];
             }
+            xdep = VS ? vd.v[0].x : z[L - 1];
         }
         if (i + 1 < pos.nrows) {
 #pragma unroll
             for (int tt = 0; tt < L; ++tt)
-                V::copy_async(xring + tt * NT, xrow + rX + (int64_t)tt * sX, 1, z[L - 1]);
+                V::copy_async(xring + tt * NT, xrow + rX + (int64_t)tt * sX, 1, xdep);
         }
         cp_async_commit();
 
         // phase 2: the soma forward, then dL/dV^s backwards in time (dL/dZ = dL/dV^s)
         float dz[L];
         {
-            float v = 0.f;
-            bool s = false;
+            if constexpr (!VS) {
+                float v = 0.f;
+                bool s = false;
 #pragma unroll
-            for (int tt = 0; tt < L; ++tt) {
-                v = soma_charge(z[tt], v, s, P);
-                s = v >= P.theta;
-                z[tt] = v;                       // z now holds V^s
+                for (int tt = 0; tt < L; ++tt) {
+                    v = soma_charge(z[tt], v, s, P);
+                    s = v >= P.theta;
+                    z[tt] = v;                   // z now holds V^s
+                }
             }
             float dvn = 0.f;                     // dL/dV^s[t+1]
 #pragma unroll
@@ -1816,6 +1876,11 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
         // the next row's dL/dS: into the ring once phase 2 has read it (dz[0] depends on
         // every read), else into the registers
         if (i + 1 < pos.nrows) {
+            if constexpr (VS) {
+#pragma unroll
+                for (int tt = 0; tt < L; ++tt)
+                    cp_async<4>(vring + tt * NT, vsrow + jstep + (int64_t)tt * BN, dz[0]);
+            }
             if constexpr (GSA) {
 #pragma unroll
                 for (int tt = 0; tt < L; ++tt)
@@ -1858,6 +1923,7 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
         gsrow += jstep;
         gxrow += rX;
         if (has_gv) gvrow += jstep;
+        if constexpr (VS) vsrow += jstep;
     }
 
     constexpr int NA1 = NA + 1;
@@ -2243,17 +2309,22 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s, int *r
     constexpr bool kPhased = DENDSN_BWD_PHASED && LAYOUT == 0 && G == 1 && K == 8 && KT == K &&
                              XI::kAsync;
     if constexpr (kPhased) {
-        if (a.g.T == L && !a.p.residual) {
-            // dL/dS by cp.async needs 4-byte words that stay inside each step's row; both
-            // builds reserve its shared memory, so the residency query (gs unknown) holds
+        if (takes_phased_backward(K, G, KT, LAYOUT, a.g.T, L, a.p.residual != 0)) {
+            // dL/dS by cp.async needs 4-byte words that stay inside each step's row; every
+            // build reserves the dL/dS and V^s rings, so the residency query (gs and the
+            // saved V^s unknown) holds for all of them
             const bool gsa = (reinterpret_cast<uintptr_t>(a.gs) & 3) == 0 && (XT == 0 || a.g.BN % 2 == 0);
-            const size_t ph = sizeof(float) * KT * L * NT + xraw * L * NT + sizeof(uint32_t) * L * NT;
+            const bool vs = gsa && a.vs_saved != nullptr;
+            const size_t ph = sizeof(float) * KT * L * NT + xraw * L * NT + 2 * sizeof(uint32_t) * L * NT;
             const size_t psm = (red > ph ? red : ph) + kappa_smem_bytes(a.p.mask_mode, KT, NT);
+            if (vs)
+                return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true, true, true>, psm)
+                                   : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false, true, true>, psm);
             if (gsa)
-                return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true, true>, psm)
-                                   : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false, true>, psm);
-            return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true, false>, psm)
-                               : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false, false>, psm);
+                return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true, true, false>, psm)
+                                   : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false, true, false>, psm);
+            return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true, false, false>, psm)
+                               : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false, false, false>, psm);
         }
     }
     // full chunks: deeper conv layer 906 -> 738 us, event layer 1829 -> 1755 us, conv layer

@@ -19,6 +19,14 @@ constexpr int lane_compartments(int K) { return K < 8 ? K : 8; }
 constexpr int bwd_lane_compartments(int K, int G, int xt, int L) {
     return (K >= 8 && G == 1 && xt == 0 && L <= 4) ? 4 : lane_compartments(K);
 }
+// Whether the backward takes the phased kernel: rows of one full chunk (T == L) of whole
+// 8-compartment neurons (one lane each), one compartment per branch, compartments
+// innermost, no residual term. The forward of such a layer keeps V^s for it when the
+// caller provides the saved buffer.
+constexpr bool takes_phased_backward(int K, int G, int KT_bwd, int layout, int T, int L,
+                                     bool residual) {
+    return K == 8 && G == 1 && KT_bwd == 8 && layout == 0 && T == L && !residual;
+}
 // Threads per block: the forward always 256; the backward 128 when a lane owns 8
 // compartments (its ~165 registers allow three 128-thread blocks per SM).
 constexpr int fwd_threads(int K) { return 256; }
@@ -58,6 +66,7 @@ struct FwdArgs {
     float *v_out;
     float *ck_vd;   // [n_ck][BN][K]  or NULL (no checkpoints written)
     float *ck_vs;   // [n_ck][BN]
+    float *vs_keep; // [T][BN] V^s for a single-chunk backward (layers with keeps_vs), or NULL
 };
 
 struct BwdArgs {
@@ -68,6 +77,7 @@ struct BwdArgs {
     const float *gv;
     const float *ck_vd;
     const float *ck_vs;
+    const float *vs_saved;   // [T][BN] V^s the forward kept (vs_keep), or NULL: recomputed
     void *gx;
     float *partials;   // [nCT * nRG][nch_max][NP], NP = 2K + 2Kb + 1 (alpha, xi, zeta, kappa, beta)
     int32_t want_beta; // accumulate the beta slot (else it stays zero)

@@ -204,12 +204,26 @@ def run_gpu(w, inp_dev: dict, gs, gv, want_v=True):
                             inp_dev["kappa"], inp_dev["mask"], want_v=False, saved=saved2)
     torch.cuda.synchronize()
     assert torch.equal(s, s2), "forward without V^s output changed the spikes"
-    if saved is not None:
+    n_ck = (w.T + 7) // 8 - 1
+    if saved is not None and n_ck > 0:
         # checkpoints: (ceil(T/8) - 1) x B*N x (K + 1) float32; the rest is alignment padding
-        n_ck = (w.T + 7) // 8 - 1
         used = n_ck * w.B * w.N * (w.K + 1) * 4
         assert torch.equal(saved[:used], saved2[:used]), \
             "forward without V^s output changed the checkpoints"
+    elif saved is not None:
+        # a layer of the phased backward: saved holds V^s [T, B, N] float32, kept by both
+        # forwards bit for bit, equal to the V^s output
+        used = w.T * w.B * w.N * 4
+        assert torch.equal(saved[:used], saved2[:used]), "the two forwards kept different V^s"
+        if v is not None:
+            assert torch.equal(saved[:used].view(torch.float32).view(v.shape), v), \
+                "the kept V^s is not the V^s output"
+    if n_ck == 0:
+        # without the saved buffer the backward recomputes everything from x: same bits
+        g1 = binding.backward(cfg, inp_dev["x"], inp_dev["alpha"], inp_dev["xi"], inp_dev["zeta"],
+                              inp_dev["kappa"], inp_dev["mask"], gs, gv, None, scratch)
+        for k in g0:
+            assert torch.equal(g0[k], g1[k]), f"{k} differs without the saved buffer"
     out = {"s": oracle.to_f64(s), "v": None if v is None else oracle.to_f64(v)}
     out.update({k: oracle.to_f64(t) for k, t in g.items()})
     return out
