@@ -314,9 +314,10 @@ dendsn_status make_plan(const dendsn_config *cfg, Plan *pl) {
     }
     pl->ck_vd_bytes = (size_t)g.n_ck * (size_t)BN * c.K * sizeof(float);
     pl->saved_bytes = pl->ck_vd_bytes + (size_t)g.n_ck * (size_t)BN * sizeof(float);
-    // rows of one chunk of whole 8-compartment neurons (the phased backward): the forward
-    // keeps V^s, so that the backward recomputes only the compartment scan
-    pl->keep_vs = takes_phased_backward(c.K, c.G, KTB, pl->layout, c.T, g.L, c.residual != 0);
+    // bfloat16 rows of one chunk of whole 8-compartment neurons (the phased backward): the
+    // forward keeps V^s, so that the backward recomputes only the compartment scan
+    pl->keep_vs = c.x_dtype == DENDSN_BF16 &&
+                  takes_phased_backward(c.K, c.G, KTB, pl->layout, c.T, g.L, c.residual != 0);
     if (pl->keep_vs) pl->saved_bytes = (size_t)c.T * (size_t)BN * sizeof(float);
     pl->saved_bytes = (pl->saved_bytes + 15) / 16 * 16;
     return DENDSN_OK;

@@ -945,7 +945,7 @@ dendsn_forward_kernel(const FwdArgs A) {
     float *vrow = A.v_out ? A.v_out + j0 : nullptr;
     // the kept V^s arises only for layers of the phased backward (one 8-compartment lane per
     // neuron, compartments innermost); elsewhere krow is null at compile time
-    constexpr bool can_keep = K == 8 && G == 1 && LAYOUT == 0;
+    constexpr bool can_keep = K == 8 && G == 1 && LAYOUT == 0 && std::is_same<XT, __nv_bfloat16>::value;
     float *krow = (can_keep && A.vs_keep) ? A.vs_keep + j0 : nullptr;
     const bool write_ck = (A.ck_vd != nullptr) && g.n_ck > 0 && pos.active;
     const bool store = pos.active && pos.sub == 0;
@@ -1720,11 +1720,7 @@ dendsn_backward_kernel(const BwdArgs A) {
 // x two rows ahead too, 529 us). For bfloat16 each thread copies the aligned 4-byte word
 // holding its element and its neighbour's; the launcher takes this build only when those
 // words lie inside each step's row (gs 4-byte aligned, B*N even), else the register one.
-// VS: V^s comes from the forward (A.vs_saved, by cp.async with dL/dS) instead of being
-// recomputed: phase 1 then only rescans V^d and phase 2 starts at the reverse recursion
-// (deeper conv backward 515.9 -> 461.8 us, for a forward that writes 4 more bytes per
-// neuron-step).
-template <int K, int PSI, typename XT, int L, bool BETA, bool GSA, bool VS>
+template <int K, int PSI, typename XT, int L, bool BETA, bool GSA>
 __global__ void __launch_bounds__(bwd_threads(K), bwd_threads(K) == 128 ? DENDSN_PHASED_MINB : 2)
 dendsn_backward_phased_kernel(const BwdArgs A) {
     constexpr int KT = K;
@@ -1736,7 +1732,6 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
     using AR = Arith<KT, 1, PSI, XT>;
     using XRaw = typename V::Raw;
     static_assert(KT % 2 == 0 && AR::KTb == KT, "paired engine only");
-    static_assert(!VS || GSA, "the kept V^s arrives with dL/dS");
     const Geometry &g = A.g;
     const Params &P = A.p;
     const ThreadPos pos = thread_pos<1>(g);
@@ -1769,9 +1764,6 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
     uint32_t *const gring = reinterpret_cast<uint32_t *>(reinterpret_cast<char *>(sregion) +
                                                          sizeof(float2) * L * N2 * NT +
                                                          sizeof(XRaw) * L * NT) + threadIdx.x;
-    // VS: the kept V^s of a row [L][NT] after the dL/dS ring
-    float *const vring = reinterpret_cast<float *>(gring + L * NT);
-    const float *vsrow = VS ? A.vs_saved + j0 : nullptr;
     auto gs_word = [&](const XT *p) {
         return reinterpret_cast<const uint32_t *>(reinterpret_cast<uintptr_t>(p) & ~(uintptr_t)3);
     };
@@ -1786,10 +1778,6 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
         if constexpr (GSA) {
 #pragma unroll
             for (int tt = 0; tt < L; ++tt) cp_async<4>(gring + tt * NT, gs_word(gsrow + (int64_t)tt * BN), 0.f);
-        }
-        if constexpr (VS) {
-#pragma unroll
-            for (int tt = 0; tt < L; ++tt) cp_async<4>(vring + tt * NT, vsrow + (int64_t)tt * BN, 0.f);
         }
     }
     cp_async_commit();
@@ -1811,8 +1799,7 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
 
         // phase 1: recompute
         cp_async_wait<0>();
-        float z[L];                              // Z, then V^s (VS: V^s from the start)
-        float xdep;                              // depends on every read of the x ring
+        float z[L];
         {
             typename AR::St vd;
             AR::zero(vd);
@@ -1820,38 +1807,28 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
             for (int tt = 0; tt < L; ++tt) {
                 float xv[KT];
                 V::unpack(xring[tt * NT], xv);
-                if constexpr (VS) {
-#pragma unroll
-                    for (int m = 0; m < N2; ++m)
-                        vd.v[m] = ffma2(lp.a[m], vd.v[m], make_float2(xv[2 * m], xv[2 * m + 1]));
-                    z[tt] = vring[tt * NT];
-                } else {
-                    z[tt] = AR::step(lp, vd, xv, false, 0.f);
-                }
+                z[tt] = AR::step(lp, vd, xv, false, 0.f);
 #pragma unroll
                 for (int m = 0; m < N2; ++m) hist[(tt * N2 + m) * NT] = vd.v[m];
             }
-            xdep = VS ? vd.v[0].x : z[L - 1];
         }
         if (i + 1 < pos.nrows) {
 #pragma unroll
             for (int tt = 0; tt < L; ++tt)
-                V::copy_async(xring + tt * NT, xrow + rX + (int64_t)tt * sX, 1, xdep);
+                V::copy_async(xring + tt * NT, xrow + rX + (int64_t)tt * sX, 1, z[L - 1]);
         }
         cp_async_commit();
 
         // phase 2: the soma forward, then dL/dV^s backwards in time (dL/dZ = dL/dV^s)
         float dz[L];
         {
-            if constexpr (!VS) {
-                float v = 0.f;
-                bool s = false;
+            float v = 0.f;
+            bool s = false;
 #pragma unroll
-                for (int tt = 0; tt < L; ++tt) {
-                    v = soma_charge(z[tt], v, s, P);
-                    s = v >= P.theta;
-                    z[tt] = v;                   // z now holds V^s
-                }
+            for (int tt = 0; tt < L; ++tt) {
+                v = soma_charge(z[tt], v, s, P);
+                s = v >= P.theta;
+                z[tt] = v;                       // z now holds V^s
             }
             float dvn = 0.f;                     // dL/dV^s[t+1]
 #pragma unroll
@@ -1876,11 +1853,6 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
         // the next row's dL/dS: into the ring once phase 2 has read it (dz[0] depends on
         // every read), else into the registers
         if (i + 1 < pos.nrows) {
-            if constexpr (VS) {
-#pragma unroll
-                for (int tt = 0; tt < L; ++tt)
-                    cp_async<4>(vring + tt * NT, vsrow + jstep + (int64_t)tt * BN, dz[0]);
-            }
             if constexpr (GSA) {
 #pragma unroll
                 for (int tt = 0; tt < L; ++tt)
@@ -1923,7 +1895,191 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
         gsrow += jstep;
         gxrow += rX;
         if (has_gv) gvrow += jstep;
-        if constexpr (VS) vsrow += jstep;
+    }
+
+    constexpr int NA1 = NA + 1;
+    float v[NA1];
+    AR::acc_export(lp, acc, v);
+    v[NA] = BETA ? gbeta : 0.f;
+#pragma unroll
+    for (int a = 0; a < NA1; ++a)
+        if (!pos.active || (a < KT && P.stateless)) v[a] = 0.f;
+    cp_async_wait<0>();
+    block_partials<KT, 1, 1, NT>(g, pos, v, reinterpret_cast<float *>(sregion), A.partials);
+}
+
+// ---------------------------------------------------------------- phased backward, kept V^s
+// dendsn_backward_phased_kernel for bfloat16 layers whose forward kept V^s (A.vs_saved).
+// The soma needs no recompute, so a row runs in three phases and V^d never goes to shared
+// memory:
+//   2. the soma's reverse recursion from the kept V^s and dL/dS (both by cp.async, one row
+//      ahead) gives dL/dZ[t] (Eqs. methods-lif-reset-charge, methods-lif-fire, methods-sg);
+//   3. pair by pair: the pair's inputs of the row from the x ring, the compartment scan
+//      forward into registers (Eq. methods-compartment), then the dendritic reverse scan
+//      (the per-pair step of dendsn_backward_kernel), dL/dX of the pair to shared memory;
+//   4. each step's dL/dX gathered and stored as one vector.
+// x arrives two rows ahead (a row's x is read until its phase 3 ends, so the ring holds
+// two rows). V^d, the accumulators and dL/dX see the same operations in the same order as
+// in dendsn_backward_phased_kernel: both give the same bits. The forward pays 4 bytes per
+// neuron-step for V^s (deeper conv forward 209 -> 230 us); the deeper conv backward went
+// 516.5 -> 471.8 us with the kept V^s in the phased kernel's four phases, and to 442.9 us
+// in these three.
+template <int K, int PSI, int L, bool BETA>
+__global__ void __launch_bounds__(bwd_threads(K), 3)
+dendsn_backward_phased_vs_kernel(const BwdArgs A) {
+    using XT = __nv_bfloat16;
+    constexpr int KT = K;
+    constexpr int NT = bwd_threads(KT);
+    constexpr int N2 = KT / 2;
+    constexpr int NA = acc_count<KT, 1>();
+    using V = XIO<XT, KT, 0>;
+    using AR = Arith<KT, 1, PSI, XT>;
+    using XRaw = typename V::Raw;
+    static_assert(KT == 8 && NT == 128 && sizeof(XRaw) == 16 && AR::KTb == KT,
+                  "one lane of 8 bfloat16 compartments per neuron");
+    const Geometry &g = A.g;
+    const Params &P = A.p;
+    const ThreadPos pos = thread_pos<1>(g);
+    typename AR::LP lp;
+    AR::load(P, g, pos.chan, 0, lp);
+    const int64_t sX = g.BN * K;
+    const int64_t BN = g.BN;
+    const int64_t j0 = pos.row0 * g.P + pos.p;
+    const int64_t jstep = (int64_t)pos.rstride * g.P;
+    const int64_t rX = jstep * K;
+    const XT *__restrict__ xrow = static_cast<const XT *>(A.x) + j0 * K;
+    const XT *__restrict__ gsrow = static_cast<const XT *>(A.gs) + j0;
+    const float *__restrict__ vsrow = A.vs_saved + j0;
+    XT *__restrict__ gxrow = static_cast<XT *>(A.gx) + j0 * K;
+    const float *gvrow = A.gv ? A.gv + j0 : nullptr;
+    const float kv = (P.detach || P.soft) ? 0.f : -P.beta;
+    const float cs = (P.detach || !P.soft) ? 0.f : -P.beta * P.theta;
+    const float b_spike = P.soft ? P.beta : 0.f;
+    const bool has_gv = A.gv != nullptr;
+    const int nrows = pos.nrows;
+
+    // dynamic shared memory: the lanes' kappa (per-neuron masks only), then dL/dX
+    // [L][N2][NT] float2, the x ring [2][L][NT], dL/dS words [L][NT] and V^s [L][NT], or (at
+    // the end) the reduction
+    extern __shared__ float4 smem_f4[];
+    char *const sregion = reinterpret_cast<char *>(smem_f4) + kappa_smem_bytes(P.mask_mode, KT, NT);
+    float2 *const gxb = reinterpret_cast<float2 *>(sregion) + threadIdx.x;
+    XRaw *const xring = reinterpret_cast<XRaw *>(reinterpret_cast<float2 *>(sregion) + L * N2 * NT) +
+                        threadIdx.x;
+    uint32_t *const gring = reinterpret_cast<uint32_t *>(sregion + sizeof(float2) * L * N2 * NT +
+                                                         sizeof(XRaw) * 2 * L * NT) + threadIdx.x;
+    float *const vring = reinterpret_cast<float *>(gring + L * NT);
+    // the aligned 4-byte word of dL/dS holding the thread's element (the launcher checks
+    // that it lies inside the step's row), and the byte selector that moves the element
+    // to the top half (exact)
+    auto gs_word = [&](const XT *p) {
+        return reinterpret_cast<const uint32_t *>(reinterpret_cast<uintptr_t>(p) & ~(uintptr_t)3);
+    };
+    auto gs_sel = [&](const XT *p) -> uint32_t {
+        return ((reinterpret_cast<uintptr_t>(p) >> 1) & 1) ? 0x3244u : 0x1044u;
+    };
+    auto fetch_x = [&](int slot, const XT *p, float dep) {
+#pragma unroll
+        for (int tt = 0; tt < L; ++tt) V::copy_async(xring + (slot * L + tt) * NT, p + (int64_t)tt * sX, 1, dep);
+    };
+    auto fetch_gv = [&](const XT *gp, const float *vp, float dep) {
+#pragma unroll
+        for (int tt = 0; tt < L; ++tt) {
+            cp_async<4>(gring + tt * NT, gs_word(gp + (int64_t)tt * BN), dep);
+            cp_async<4>(vring + tt * NT, vp + (int64_t)tt * BN, dep);
+        }
+    };
+    // commit pattern: rows 0 (x, dL/dS, V^s) and 1 (x); then per row i, after phase 2 the
+    // next row's dL/dS and V^s, after phase 3 the x of row i + 2. A row waits for all but the
+    // newest group.
+    if (nrows > 0) {
+        fetch_x(0, xrow, 0.f);
+        fetch_gv(gsrow, vsrow, 0.f);
+    }
+    cp_async_commit();
+    if (nrows > 1) fetch_x(1, xrow + rX, 0.f);
+    cp_async_commit();
+
+    typename AR::Acc acc;
+    AR::acc_zero(acc);
+    float gbeta = 0.f;
+    MaskAhead<AR, NT> mask;
+    mask.init(P, g, j0, jstep, pos.chan, 0, nrows, smem_f4);
+    for (int i = 0; i < nrows; ++i) {
+        mask.advance(P, g, 0, i + 1 < nrows, lp);
+        cp_async_wait<1>();
+
+        // phase 2: dL/dV^s backwards in time from the kept V^s (dL/dZ = dL/dV^s)
+        float dz[L];
+        {
+            const uint32_t sel = gs_sel(gsrow);
+            float dvn = 0.f;                     // dL/dV^s[t+1]
+#pragma unroll
+            for (int tt = L - 1; tt >= 0; --tt) {
+                const float vs = vring[tt * NT];
+                const bool st = vs >= P.theta;
+                if constexpr (BETA) {
+                    const float leak = st ? (P.soft ? __fsub_rn(vs, P.theta) : 0.f) : vs;
+                    gbeta = __fmaf_rn(dvn, leak, gbeta);
+                }
+                const float dvds = __fmaf_rn(kv, vs, cs);
+                const float dvdv = st ? b_spike : P.beta;
+                const float gst = __uint_as_float(__byte_perm(gring[tt * NT], 0u, sel));
+                const float ds = __fmaf_rn(dvds, dvn, gst);
+                float dv = __fmaf_rn(surrogate(__fsub_rn(vs, P.theta)), ds, __fmul_rn(dvdv, dvn));
+                if (has_gv) dv = __fadd_rn(dv, __ldcs(gvrow + (int64_t)tt * BN));
+                dz[tt] = dv;
+                dvn = dv;
+            }
+        }
+        // the next row's dL/dS and V^s, once phase 2 has read them (dz[0] depends on every read)
+        if (i + 1 < nrows) fetch_gv(gsrow + jstep, vsrow + jstep, dz[0]);
+        cp_async_commit();
+
+        // phase 3: per compartment pair, V^d forward into registers, then the reverse scan
+        const XRaw *xs = xring + (i & 1) * L * NT;
+#pragma unroll
+        for (int m = 0; m < N2; ++m) {
+            float2 vd[L];
+            float2 v = f2(0.f);
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) {
+                const uint32_t w = reinterpret_cast<const uint32_t *>(xs + tt * NT)[m];
+                v = ffma2(lp.a[m], v, make_float2(bf16_lo(w), bf16_hi(w)));
+                vd[tt] = v;
+            }
+            float2 Ad = f2(0.f);
+#pragma unroll
+            for (int tt = L - 1; tt >= 0; --tt)
+                gxb[(tt * N2 + m) * NT] = AR::pair_back(lp, m, vd[tt], tt > 0 ? vd[tt > 0 ? tt - 1 : 0] : f2(0.f),
+                                                        f2(-dz[tt]), f2(0.f), Ad, acc);
+        }
+        // x of row i + 2 into the slot just read (the sum depends on every pair's reads)
+        if (i + 2 < nrows) {
+            const float dep = __fadd_rn(__fadd_rn(acc.ga[0].x, acc.ga[1].x), __fadd_rn(acc.ga[2].x, acc.ga[3].x));
+            fetch_x(i & 1, xrow + 2 * rX, dep);
+        }
+        cp_async_commit();
+
+        // phase 4: dL/dX of each step as one vector
+        if (pos.active) {
+#pragma unroll
+            for (int tt = 0; tt < L; ++tt) {
+                float gxv[KT];
+#pragma unroll
+                for (int m = 0; m < N2; ++m) {
+                    const float2 q = gxb[(tt * N2 + m) * NT];
+                    gxv[2 * m] = q.x;
+                    gxv[2 * m + 1] = q.y;
+                }
+                V::store(gxrow + (int64_t)tt * sX, 1, gxv);
+            }
+        }
+        xrow += rX;
+        gsrow += jstep;
+        vsrow += jstep;
+        gxrow += rX;
+        if (has_gv) gvrow += jstep;
     }
 
     constexpr int NA1 = NA + 1;
@@ -2310,21 +2466,25 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s, int *r
                              XI::kAsync;
     if constexpr (kPhased) {
         if (takes_phased_backward(K, G, KT, LAYOUT, a.g.T, L, a.p.residual != 0)) {
-            // dL/dS by cp.async needs 4-byte words that stay inside each step's row; every
-            // build reserves the dL/dS and V^s rings, so the residency query (gs and the
-            // saved V^s unknown) holds for all of them
+            // dL/dS by cp.async needs 4-byte words that stay inside each step's row; the
+            // recompute build reserves its shared memory either way, so the residency query
+            // (gs unknown) holds for both. (The kept-V^s kernel fits the same 3 blocks per SM.)
             const bool gsa = (reinterpret_cast<uintptr_t>(a.gs) & 3) == 0 && (XT == 0 || a.g.BN % 2 == 0);
-            const bool vs = gsa && a.vs_saved != nullptr;
-            const size_t ph = sizeof(float) * KT * L * NT + xraw * L * NT + 2 * sizeof(uint32_t) * L * NT;
+            if constexpr (XT == 1) {
+                if (gsa && a.vs_saved != nullptr) {
+                    const size_t vb = sizeof(float) * KT * L * NT + xraw * 2 * L * NT + 2 * sizeof(uint32_t) * L * NT;
+                    const size_t vsm = (red > vb ? red : vb) + kappa_smem_bytes(a.p.mask_mode, KT, NT);
+                    return a.want_beta ? go_smem(dendsn_backward_phased_vs_kernel<K, PSI, L, true>, vsm)
+                                       : go_smem(dendsn_backward_phased_vs_kernel<K, PSI, L, false>, vsm);
+                }
+            }
+            const size_t ph = sizeof(float) * KT * L * NT + xraw * L * NT + sizeof(uint32_t) * L * NT;
             const size_t psm = (red > ph ? red : ph) + kappa_smem_bytes(a.p.mask_mode, KT, NT);
-            if (vs)
-                return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true, true, true>, psm)
-                                   : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false, true, true>, psm);
             if (gsa)
-                return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true, true, false>, psm)
-                                   : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false, true, false>, psm);
-            return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true, false, false>, psm)
-                               : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false, false, false>, psm);
+                return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true, true>, psm)
+                                   : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false, true>, psm);
+            return a.want_beta ? go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, true, false>, psm)
+                               : go_smem(dendsn_backward_phased_kernel<K, PSI, T, L, false, false>, psm);
         }
     }
     // full chunks: deeper conv layer 906 -> 738 us, event layer 1829 -> 1755 us, conv layer

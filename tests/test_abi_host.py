@@ -112,17 +112,17 @@ def test_workspace_sizes_follow_checkpoint_layout():
     for T in (1, 4, 5, 8):
         saved, scratch = binding.dendsn_workspace_size(make_config(T=T, B=2, N=256, K=4, C=2, inner=128))
         assert saved == 0 and scratch > 0
-    # rows of one chunk of whole 8-compartment neurons (the phased backward): the forward
-    # keeps V^s, T x B x N float32
+    # bfloat16 rows of one chunk of whole 8-compartment neurons (the phased backward): the
+    # forward keeps V^s, T x B x N float32
     B, N = 3, 256
-    for T, dt in ((8, "f32"), (8, "bf16"), (4, "bf16")):
+    for T, dt in ((8, "bf16"), (4, "bf16")):
         saved, _ = binding.dendsn_workspace_size(make_config(T=T, B=B, N=N, K=8, C=2, inner=128,
                                                              dtype=dt))
         assert saved == T * B * N * 4, (T, dt)
-    # not that backward: float32 T = 4 (split lanes), T between chunk lengths, the residual
-    # term, the paper layout, two compartments per branch
-    for kw in (dict(T=4), dict(T=6, dtype="bf16"), dict(T=8, residual=True),
-               dict(T=8, layout="paper"), dict(T=8, G=2)):
+    # not those layers: float32 (T = 8 phased without a kept V^s; T = 4 split lanes), T
+    # between chunk lengths, the residual term, the paper layout, two compartments per branch
+    for kw in (dict(T=8), dict(T=4), dict(T=6, dtype="bf16"), dict(T=8, dtype="bf16", residual=True),
+               dict(T=8, dtype="bf16", layout="paper"), dict(T=8, dtype="bf16", G=2)):
         saved, _ = binding.dendsn_workspace_size(make_config(**dict(dict(B=B, N=N, K=8, C=2,
                                                                          inner=128), **kw)))
         assert saved == 0, kw
