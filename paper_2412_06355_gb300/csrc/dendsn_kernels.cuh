@@ -1923,7 +1923,8 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
 // in dendsn_backward_phased_kernel: both give the same bits. The forward pays 4 bytes per
 // neuron-step for V^s (deeper conv forward 209 -> 230 us); the deeper conv backward went
 // 516.5 -> 471.8 us with the kept V^s in the phased kernel's four phases, and to 442.9 us
-// in these three.
+// in these three. Reading x as 8-byte halves (two pairs) instead of each pair's 4-byte
+// word (a 4-way bank conflict) measured slower: 442.8 -> 488.3 us (more live registers).
 template <int K, int PSI, int L, bool BETA>
 __global__ void __launch_bounds__(bwd_threads(K), 3)
 dendsn_backward_phased_vs_kernel(const BwdArgs A) {
@@ -1958,16 +1959,17 @@ dendsn_backward_phased_vs_kernel(const BwdArgs A) {
     const bool has_gv = A.gv != nullptr;
     const int nrows = pos.nrows;
 
-    // dynamic shared memory: the lanes' kappa (per-neuron masks only), then dL/dX
-    // [L][N2][NT] float2, the x ring [2][L][NT], dL/dS words [L][NT] and V^s [L][NT], or (at
-    // the end) the reduction
+    // dynamic shared memory: the lanes' kappa (per-neuron masks only), then dL/dX as packed
+    // bfloat16 pairs [L][N2][NT] (half the shared-memory traffic of float pairs: 442.6 ->
+    // 428.8 us), the x ring [2][L][NT], dL/dS words [L][NT] and V^s [L][NT], or (at the end)
+    // the reduction
     extern __shared__ float4 smem_f4[];
     char *const sregion = reinterpret_cast<char *>(smem_f4) + kappa_smem_bytes(P.mask_mode, KT, NT);
-    float2 *const gxb = reinterpret_cast<float2 *>(sregion) + threadIdx.x;
-    XRaw *const xring = reinterpret_cast<XRaw *>(reinterpret_cast<float2 *>(sregion) + L * N2 * NT) +
-                        threadIdx.x;
-    uint32_t *const gring = reinterpret_cast<uint32_t *>(sregion + sizeof(float2) * L * N2 * NT +
-                                                         sizeof(XRaw) * 2 * L * NT) + threadIdx.x;
+    uint32_t *const gxw = reinterpret_cast<uint32_t *>(sregion) + threadIdx.x;
+    constexpr size_t GXB = sizeof(uint32_t) * L * N2 * NT;
+    XRaw *const xring = reinterpret_cast<XRaw *>(sregion + GXB) + threadIdx.x;
+    uint32_t *const gring = reinterpret_cast<uint32_t *>(sregion + GXB + sizeof(XRaw) * 2 * L * NT) +
+                            threadIdx.x;
     float *const vring = reinterpret_cast<float *>(gring + L * NT);
     // the aligned 4-byte word of dL/dS holding the thread's element (the launcher checks
     // that it lies inside the step's row), and the byte selector that moves the element
@@ -2050,9 +2052,11 @@ dendsn_backward_phased_vs_kernel(const BwdArgs A) {
             }
             float2 Ad = f2(0.f);
 #pragma unroll
-            for (int tt = L - 1; tt >= 0; --tt)
-                gxb[(tt * N2 + m) * NT] = AR::pair_back(lp, m, vd[tt], tt > 0 ? vd[tt > 0 ? tt - 1 : 0] : f2(0.f),
-                                                        f2(-dz[tt]), f2(0.f), Ad, acc);
+            for (int tt = L - 1; tt >= 0; --tt) {
+                const float2 gq = AR::pair_back(lp, m, vd[tt], tt > 0 ? vd[tt > 0 ? tt - 1 : 0] : f2(0.f),
+                                                f2(-dz[tt]), f2(0.f), Ad, acc);
+                gxw[(tt * N2 + m) * NT] = pack_bf16x2(gq.x, gq.y);
+            }
         }
         // x of row i + 2 into the slot just read (the sum depends on every pair's reads)
         if (i + 2 < nrows) {
@@ -2065,14 +2069,9 @@ dendsn_backward_phased_vs_kernel(const BwdArgs A) {
         if (pos.active) {
 #pragma unroll
             for (int tt = 0; tt < L; ++tt) {
-                float gxv[KT];
-#pragma unroll
-                for (int m = 0; m < N2; ++m) {
-                    const float2 q = gxb[(tt * N2 + m) * NT];
-                    gxv[2 * m] = q.x;
-                    gxv[2 * m + 1] = q.y;
-                }
-                V::store(gxrow + (int64_t)tt * sX, 1, gxv);
+                __stcs(reinterpret_cast<uint4 *>(gxrow + (int64_t)tt * sX),
+                       make_uint4(gxw[(tt * N2 + 0) * NT], gxw[(tt * N2 + 1) * NT],
+                                  gxw[(tt * N2 + 2) * NT], gxw[(tt * N2 + 3) * NT]));
             }
         }
         xrow += rX;
@@ -2472,7 +2471,8 @@ cudaError_t launch_backward(const BwdArgs &a, int blocks, cudaStream_t s, int *r
             const bool gsa = (reinterpret_cast<uintptr_t>(a.gs) & 3) == 0 && (XT == 0 || a.g.BN % 2 == 0);
             if constexpr (XT == 1) {
                 if (gsa && a.vs_saved != nullptr) {
-                    const size_t vb = sizeof(float) * KT * L * NT + xraw * 2 * L * NT + 2 * sizeof(uint32_t) * L * NT;
+                    const size_t vb = sizeof(uint32_t) * (KT / 2) * L * NT + xraw * 2 * L * NT +
+                                      2 * sizeof(uint32_t) * L * NT;
                     const size_t vsm = (red > vb ? red : vb) + kappa_smem_bytes(a.p.mask_mode, KT, NT);
                     return a.want_beta ? go_smem(dendsn_backward_phased_vs_kernel<K, PSI, L, true>, vsm)
                                        : go_smem(dendsn_backward_phased_vs_kernel<K, PSI, L, false>, vsm);
