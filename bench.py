@@ -158,8 +158,10 @@ def kernel_names(w):
     narrow long-horizon layers take the time-parallel kernels; rows of one full chunk
     (T = 4 or 8) whose 8 compartments sit on one lane, compartments innermost and no
     residual term, take the phased backward (one lane per neuron: bf16, or float32 with
-    8-step chunks); 4-step rows of 8 float32 compartments on two lanes (no residual term,
-    either layout) the row-pair backward; the rest the chunked kernels."""
+    8-step chunks; for bf16 the build that reads the V^s its forward kept in the saved
+    buffer, which the benchmark always provides); 4-step rows of 8 float32 compartments on
+    two lanes (no residual term, either layout) the row-pair backward; the rest the chunked
+    kernels."""
     if w.T >= 256 and w.B * w.N <= 2048:
         return "tp_forward_kernel", "tp_backward_kernel"
     L = 4 if w.T <= 4 else 8
@@ -168,7 +170,8 @@ def kernel_names(w):
     fwd = "dendsn_forward_staged_kernel" if staged else "dendsn_forward_kernel"
     one_lane = w.K == 8 and w.G == 1 and (w.dtype == "bf16" or L == 8)
     if one_lane and layout0 and w.T == L and not w.residual:
-        return fwd, "dendsn_backward_phased_kernel"
+        return fwd, ("dendsn_backward_phased_vs_kernel" if w.dtype == "bf16"
+                     else "dendsn_backward_phased_kernel")
     if w.K == 8 and w.G == 1 and w.dtype == "f32" and w.T == 4 and not w.residual:
         return fwd, "dendsn_backward_rowpair_kernel"
     return fwd, "dendsn_backward_kernel"

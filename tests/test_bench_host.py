@@ -45,7 +45,8 @@ def test_kernel_names_follow_the_library_plan():
     assert bench.kernel_names(W["token_dbg"].with_(T=5))[1] == "dendsn_backward_kernel"
     assert bench.kernel_names(W["event"]) == ("dendsn_forward_kernel", "dendsn_backward_kernel")
     # rows of one full 8-step chunk, 8 bf16 compartments on one lane
-    assert bench.kernel_names(W["deepconv_bf16"])[1] == "dendsn_backward_phased_kernel"
+    assert bench.kernel_names(W["deepconv_bf16"])[1] == "dendsn_backward_phased_vs_kernel"
+    assert bench.kernel_names(W["deepconv_bf16"].with_(dtype="f32"))[1] == "dendsn_backward_phased_kernel"
     # ... but not with the residual term, nor in the paper layout
     assert bench.kernel_names(W["deepconv_bf16"].with_(residual=True))[1] == "dendsn_backward_kernel"
     assert bench.kernel_names(W["deepconv_bf16"].with_(layout="paper"))[1] == "dendsn_backward_kernel"
