@@ -267,6 +267,14 @@ __device__ __forceinline__ void load_param_arrays(const Params &P, const Geometr
         km[b] = __fmul_rn(__ldg(P.kappa + (int64_t)chan * g.Kb + sub * KTb + b), mk[b]);
 }
 
+// The lane's unmasked kappa, read once for the parameter-gradient export.
+template <int KTb>
+__device__ __forceinline__ void lane_kappa(const Params &P, const Geometry &g, int chan, int sub,
+                                           float (&kap)[KTb]) {
+#pragma unroll
+    for (int b = 0; b < KTb; ++b) kap[b] = __ldg(P.kappa + (int64_t)chan * g.Kb + sub * KTb + b);
+}
+
 // kappa * m and m for the neuron n of a per-neuron mask (mask_mode 2).
 template <int KTb>
 __device__ __forceinline__ typename MaskRaw<KTb>::T fetch_neuron_mask(const Params &P, const Geometry &g,
@@ -304,11 +312,23 @@ __host__ __device__ constexpr size_t kappa_smem_bytes(int mask_mode, int KTb, in
 // exactly 0 where m = 0 at no extra instruction; for the identity lm holds m itself. (The
 // forward needs no masked Y: kappa m = 0 already removes the branch from Z.)
 // The backward carries the dendritic adjoint and three of its sums without the factor
-// 1/zeta of Eq. methods-branch-aggregation (a per-lane constant): Ad' = zeta Ad, and
-// dL/dalpha, dL/dxi, dL/dzeta are scaled by 1/zeta once, in acc_export.
+// 1/zeta of Eq. methods-branch-aggregation (a per-lane constant): A = zeta Ad, and
+// dL/dalpha, dL/dxi, dL/dzeta are scaled by 1/zeta once, in acc_export. Lanes of 8
+// compartments (KAPPA_FREE) also leave out the factor kappa m of Eq. methods-soma-input:
+// A = zeta Ad / (kappa m), so that dL/du / (kappa m) = -dL/dZ psi'(u) enters the scan with
+// no product by kappa m; dL/dX = A (kappa m / zeta), and the three sums are scaled by
+// kappa / zeta in acc_export (a masked branch's terms are 0: its e^{-r^2/2}, or for the
+// identity its m, is 0; so the unmasked kappa scales every row, whatever the row's mask;
+// a kappa of 0 gives A finite and every scaled result 0). The phased backward forms
+// kappa m / zeta once per compartment pair and row, which saves one paired multiply per
+// pair and step (kept-V^s deeper conv backward 428.4 -> 418.4 us); the chunked backward
+// must form it every step, and with 4 compartments per lane that version spilled more
+// (conv layer 216 -> 230 us), so 4-compartment lanes keep the product by kappa m in the
+// step. Both layouts of a layer take lanes of the same width, so their bits still agree.
 template <int KT, int PSI, bool TREE>
 struct PairArith {
     static constexpr bool kTree = TREE;
+    static constexpr bool KAPPA_FREE = KT == 8;
     static constexpr int N2 = KT / 2;
     static constexpr int KTb = KT;
     struct LP { float2 a[N2], nxi[N2], iz[N2], km[N2], lm[N2]; };
@@ -450,13 +470,16 @@ struct PairArith {
             for (int q = 0; q < 4; ++q) *f[q] = make_float2(t[(8 * m + 2 * q) * NT], t[(8 * m + 2 * q + 1) * NT]);
         }
     }
-    // [alpha KT | xi KT | zeta KTb | kappa KTb]; the first three carry the factor 1/zeta here
-    static __device__ __forceinline__ void acc_export(const LP &lp, const Acc &c, float *v) {
+    // [alpha KT | xi KT | zeta KTb | kappa KTb]; the first three carry the factor 1/zeta, or
+    // kappa/zeta (KAPPA_FREE), here (kap: the lane's unmasked kappa)
+    static __device__ __forceinline__ void acc_export(const LP &lp, const Acc &c, float *v,
+                                                      const float (&kap)[KT]) {
 #pragma unroll
         for (int m = 0; m < N2; ++m) {
-            const float2 ga = fmul2(c.ga[m], lp.iz[m]);
-            const float2 gxi = fmul2(c.ngxi[m], lp.iz[m]);
-            const float2 gz = fmul2(c.ngz[m], lp.iz[m]);
+            const float2 kz = KAPPA_FREE ? fmul2(make_float2(kap[2 * m], kap[2 * m + 1]), lp.iz[m]) : lp.iz[m];
+            const float2 ga = fmul2(c.ga[m], kz);
+            const float2 gxi = fmul2(c.ngxi[m], kz);
+            const float2 gz = fmul2(c.ngz[m], kz);
             v[2 * m] = ga.x;                     v[2 * m + 1] = ga.y;
             v[KT + 2 * m] = -gxi.x;              v[KT + 2 * m + 1] = -gxi.y;
             v[2 * KT + 2 * m] = -gz.x;           v[2 * KT + 2 * m + 1] = -gz.y;
@@ -464,8 +487,8 @@ struct PairArith {
         }
     }
     // One reverse step: V^d[t] (vdt), V^d[t-1] (vdp) and dL/dZ[t] (dz) update the scaled
-    // dendritic adjoint Ad' = zeta dL/dV^d (reverse scan of Eq. methods-compartment), the
-    // parameter-gradient partials, and give dL/dX[t] = Ad' / zeta + res.
+    // dendritic adjoint A (reverse scan of Eq. methods-compartment), the parameter-gradient
+    // partials, and give dL/dX[t] + res.
     // Per branch (G = 1): dL/du = kappa m dz psi'(u) with psi'(u) = u (u^2 - 3) e^{-u^2/2}
     // (the Mexican hat of |u| is smooth in u) or sign(u) (identity); the direct term of
     // dL/dV^d is dL/du / zeta; du/dxi = -1/zeta; du/dzeta = -u / zeta.
@@ -475,39 +498,43 @@ struct PairArith {
         const float2 res2 = f2(res);
 #pragma unroll
         for (int m = 0; m < N2; ++m) {
-            const float2 g = pair_back(lp, m, vdt.v[m], vdp.v[m], ndz2, res2, Ad.v[m], acc);
+            const float2 g = pair_back(lp, m, vdt.v[m], vdp.v[m], ndz2, res2, Ad.v[m], acc,
+                                       KAPPA_FREE ? fmul2(lp.km[m], lp.iz[m]) : lp.iz[m]);
             gx[2 * m] = g.x;
             gx[2 * m + 1] = g.y;
         }
     }
-    // Pair m of one reverse step (see backward), given ndz2 = -dL/dZ[t]; returns dL/dX[t]
-    // of the pair.
+    // Pair m of one reverse step (see backward), given ndz2 = -dL/dZ[t] and the pair's
+    // kappa m / zeta (KAPPA_FREE) or 1 / zeta (kmz); returns dL/dX[t] of the pair.
     static __device__ __forceinline__ float2 pair_back(const LP &lp, int m, float2 vdt, float2 vdp,
-                                                       float2 ndz2, float2 res2, float2 &Adm, Acc &acc) {
+                                                       float2 ndz2, float2 res2, float2 &Adm, Acc &acc,
+                                                       float2 kmz) {
         {
             const float2 u = ffma2(vdt, lp.iz[m], lp.nxi[m]);
-            const float2 ngy = fmul2(lp.km[m], ndz2);            // -dL/dY
-            float2 y, du;                                        // m Y, dL/du
+            // -dL/dY, or -m dL/dZ (KAPPA_FREE)
+            const float2 ngy = fmul2(KAPPA_FREE ? lp.lm[m] : lp.km[m], ndz2);
+            float2 y, du;                                        // m Y; dL/du, or / (kappa m)
             if constexpr (PSI == PSI_MEXHAT) {
                 const float2 ss = fmul2(u, u);
                 const float2 t = ffma2(f2(kNegHalfLog2e), ss, lp.lm[m]);
                 const float2 e = make_float2(fast_exp2(t.x), fast_exp2(t.y));
                 y = ffma2(neg2(ss), e, e);
                 // psi'(r) / r = (r^2 - 3) e^{-r^2/2} = -(2 e^{-r^2/2} + psi(r)): one fused
-                // multiply-add from y; its sign cancels against that of -dL/dY
+                // multiply-add from y; its sign cancels against that of -dL/dZ
                 const float2 nw = ffma2(f2(2.f), e, y);
-                du = fmul2(nw, fmul2(u, ngy));
+                du = KAPPA_FREE ? fmul2(fmul2(nw, u), ndz2) : fmul2(nw, fmul2(u, ngy));
             } else {
                 y = fmul2(lp.lm[m], make_float2(fabsf(u.x), fabsf(u.y)));
                 du = make_float2(u.x > 0.f ? -ngy.x : (u.x < 0.f ? ngy.x : 0.f),
                                  u.y > 0.f ? -ngy.y : (u.y < 0.f ? ngy.y : 0.f));
             }
+            // (KAPPA_FREE: each of ngxi, ngz, ga times kappa)
             acc.ngxi[m] = fadd2(acc.ngxi[m], du);                // zeta dxi = -sum du
             acc.ngz[m] = ffma2(u, du, acc.ngz[m]);               // zeta dzeta = -sum u du
             acc.ngk[m] = ffma2(y, ndz2, acc.ngk[m]);             // dkappa = sum m Y dz
             Adm = ffma2(lp.a[m], Adm, du);
             acc.ga[m] = ffma2(Adm, vdp, acc.ga[m]);              // zeta dalpha
-            return ffma2(Adm, lp.iz[m], res2);
+            return ffma2(Adm, kmz, res2);
         }
     }
 };
@@ -516,6 +543,7 @@ struct PairArith {
 template <int KT, int G, int PSI>
 struct ScalarArith {
     static constexpr int KTb = KT / G;
+    static constexpr bool KAPPA_FREE = false;
     struct LP { float a[KT], nxi[KT], iz[KTb], km[KTb], mk[KTb]; };
     struct St { float v[KT]; };
     struct Acc { float ga[KT], gxi[KT], gz[KTb], gk[KTb]; };
@@ -607,7 +635,8 @@ struct ScalarArith {
 #pragma unroll
         for (int b = 0; b < KTb; ++b) { c.gz[b] = t[(2 * KT + b) * NT]; c.gk[b] = t[(2 * KT + KTb + b) * NT]; }
     }
-    static __device__ __forceinline__ void acc_export(const LP &, const Acc &c, float *v) {
+    template <int N>
+    static __device__ __forceinline__ void acc_export(const LP &, const Acc &c, float *v, const float (&)[N]) {
 #pragma unroll
         for (int i = 0; i < KT; ++i) { v[i] = c.ga[i]; v[KT + i] = c.gxi[i]; }
 #pragma unroll
@@ -1680,7 +1709,9 @@ dendsn_backward_kernel(const BwdArgs A) {
     // (slot NA: beta, counted once per neuron, by its first lane)
     constexpr int NA1 = NA + 1;
     float v[NA1];
-    AR::acc_export(lp, acc, v);
+    float kap[AR::KTb] = {};
+    if constexpr (AR::KAPPA_FREE) lane_kappa<AR::KTb>(P, g, pos.chan, pos.sub, kap);
+    AR::acc_export(lp, acc, v, kap);
     v[NA] = (BETA && pos.sub == 0) ? gbeta : 0.f;
 #pragma unroll
     for (int a = 0; a < NA1; ++a)
@@ -1867,12 +1898,13 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
         // phase 3: the dendritic reverse scan, one pair at a time
 #pragma unroll
         for (int m = 0; m < N2; ++m) {
+            const float2 kmz = fmul2(lp.km[m], lp.iz[m]);
             float2 Ad = f2(0.f);
             float2 vdt = hist[((L - 1) * N2 + m) * NT];
 #pragma unroll
             for (int tt = L - 1; tt >= 0; --tt) {
                 const float2 vdp = tt > 0 ? hist[((tt > 0 ? tt - 1 : 0) * N2 + m) * NT] : f2(0.f);
-                hist[(tt * N2 + m) * NT] = AR::pair_back(lp, m, vdt, vdp, f2(-dz[tt]), f2(0.f), Ad, acc);
+                hist[(tt * N2 + m) * NT] = AR::pair_back(lp, m, vdt, vdp, f2(-dz[tt]), f2(0.f), Ad, acc, kmz);
                 vdt = vdp;
             }
         }
@@ -1899,7 +1931,9 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
 
     constexpr int NA1 = NA + 1;
     float v[NA1];
-    AR::acc_export(lp, acc, v);
+    float kap[AR::KTb] = {};
+    if constexpr (AR::KAPPA_FREE) lane_kappa<AR::KTb>(P, g, pos.chan, 0, kap);
+    AR::acc_export(lp, acc, v, kap);
     v[NA] = BETA ? gbeta : 0.f;
 #pragma unroll
     for (int a = 0; a < NA1; ++a)
@@ -2050,11 +2084,12 @@ dendsn_backward_phased_vs_kernel(const BwdArgs A) {
                 v = ffma2(lp.a[m], v, make_float2(bf16_lo(w), bf16_hi(w)));
                 vd[tt] = v;
             }
+            const float2 kmz = fmul2(lp.km[m], lp.iz[m]);
             float2 Ad = f2(0.f);
 #pragma unroll
             for (int tt = L - 1; tt >= 0; --tt) {
                 const float2 gq = AR::pair_back(lp, m, vd[tt], tt > 0 ? vd[tt > 0 ? tt - 1 : 0] : f2(0.f),
-                                                f2(-dz[tt]), f2(0.f), Ad, acc);
+                                                f2(-dz[tt]), f2(0.f), Ad, acc, kmz);
                 gxw[(tt * N2 + m) * NT] = pack_bf16x2(gq.x, gq.y);
             }
         }
@@ -2083,7 +2118,9 @@ dendsn_backward_phased_vs_kernel(const BwdArgs A) {
 
     constexpr int NA1 = NA + 1;
     float v[NA1];
-    AR::acc_export(lp, acc, v);
+    float kap[AR::KTb] = {};
+    if constexpr (AR::KAPPA_FREE) lane_kappa<AR::KTb>(P, g, pos.chan, 0, kap);
+    AR::acc_export(lp, acc, v, kap);
     v[NA] = BETA ? gbeta : 0.f;
 #pragma unroll
     for (int a = 0; a < NA1; ++a)
