@@ -522,9 +522,13 @@ class Layer:
 
 
 def time_layer(layer, args, world, dev):
-    """Warm-up, then exactly args.steps timed steps between barriers and synchronizes.
-    Returns the per-step event times, the whole-region time (max over ranks), the wall-clock
-    window and the launch count."""
+    """Warm-up, then args.steps steps with an event pair around each step's forward and
+    backward (the split), then exactly args.steps timed steps without them, between
+    barriers and synchronizes: the layer's time. Each event record is a stream operation of
+    its own (about 2 us between two kernels, 6 us a step), instrumentation that a training
+    step does not have. Returns the per-step event times, the whole-region time of the plain
+    pass (max over ranks; and that of the instrumented pass), its wall-clock window and its
+    launch count."""
     import torch
     import torch.distributed as dist
     from paper_2412_06355_gb300 import binding, distributed
@@ -549,11 +553,22 @@ def time_layer(layer, args, world, dev):
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
+    start.record(stream)
+    for i in range(args.steps):
+        step(ev[i])
+    end.record(stream)
+    torch.cuda.synchronize()
+    ms_events = start.elapsed_time(end)
+
+    # the timed region: the same steps without the per-step event records
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
     n_launch0 = binding.launch_count()
     t0 = time.time()
     start.record(stream)
     for i in range(args.steps):
-        step(ev[i])
+        step()
     end.record(stream)
     torch.cuda.synchronize()
     t1 = time.time()
@@ -564,10 +579,10 @@ def time_layer(layer, args, world, dev):
         dist.barrier()
     ms = start.elapsed_time(end)
     if world > 1:
-        t = torch.tensor([ms], device=dev)
+        t = torch.tensor([ms, ms_events], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    return dict(ms=ms, fwd_ms=[e[0].elapsed_time(e[1]) for e in ev],
+        ms, ms_events = float(t[0].item()), float(t[1].item())
+    return dict(ms=ms, ms_events=ms_events, fwd_ms=[e[0].elapsed_time(e[1]) for e in ev],
                 bwd_ms=[e[1].elapsed_time(e[2]) for e in ev], t0=t0, t1=t1, launches=n_launch)
 
 
@@ -709,7 +724,8 @@ def layer_report(layer, timing, world, dev, peak, peak_kind, clock):
            "step_gbs": ab["total"] / (step_ms / 1e3) / 1e9,
            "frac_of_8tbs": ab["total"] / (step_ms / 1e3) / 1e9 / NOMINAL_HBM_GBS,
            "frac_of_measured": ab["total"] / (step_ms / 1e3) / 1e9 / peak,
-           "forward_ms": fwd_avg, "backward_ms": bwd_avg}
+           "forward_ms": fwd_avg, "backward_ms": bwd_avg,
+           "step_ms_with_step_events": timing["ms_events"] / layer.args.steps}
     return value, step_ms, roof, hbm
 
 
