@@ -591,11 +591,12 @@ def time_e2e(layer, args, world, dev):
 
     Each step is the headline call itself (one forward and one backward over the whole
     batch) between a host->device copy of its inputs (x, dL/dS) and a device->host copy of
-    its results (spikes, dL/dX, the parameter gradients). Two sets of device buffers
-    alternate between steps, and the copies of each direction and the kernels run on three
-    streams ordered by events, so the next step's upload overlaps this step's download. The
-    host waits for each step's results before it enqueues the step after next. Timed on the
-    wall clock."""
+    its result, the parameter gradients (what a training step hands to the optimizer; the
+    spikes and dL/dX are the tensors the next and the previous layer read on the device).
+    Two sets of device buffers alternate between steps, and the copies of each direction and
+    the kernels run on three streams ordered by events, so the next step's upload overlaps
+    this step's kernels and download. The host waits for each step's result before it
+    enqueues the step after next. Timed on the wall clock."""
     import torch
     import torch.distributed as dist
     from paper_2412_06355_gb300 import binding, distributed
@@ -607,8 +608,6 @@ def time_e2e(layer, args, world, dev):
     gs_h = torch.empty(gs.shape, dtype=gs.dtype, **pin)
     x_h.copy_(x)
     gs_h.copy_(gs)
-    s_h = torch.empty((w.T, w.B, w.N), dtype=x.dtype, **pin)
-    gx_h = torch.empty(x.shape, dtype=x.dtype, **pin)
     ng = layer.grads.numel()
     g_h = torch.empty(ng, dtype=torch.float32, **pin)
     sets = []
@@ -619,8 +618,7 @@ def time_e2e(layer, args, world, dev):
                          gx=torch.empty_like(x), ws=binding.workspace(cfg, dev), g=g_d,
                          gv=distributed.split_param_grads(g_d, w.C, w.K, w.Kb)))
     h2d = x_h.numel() * x_h.element_size() + gs_h.numel() * gs_h.element_size()
-    d2h = (s_h.numel() * s_h.element_size() + gx_h.numel() * gx_h.element_size() +
-           g_h.numel() * g_h.element_size())
+    d2h = g_h.numel() * g_h.element_size()
     up, comp, down = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
     ev = lambda: torch.cuda.Event()                   # noqa: E731
     loaded, computed, returned = ([ev(), ev()] for _ in range(3))
@@ -646,8 +644,6 @@ def time_e2e(layer, args, world, dev):
         computed[i].record(comp)
         with torch.cuda.stream(down):
             down.wait_event(computed[i])
-            s_h.copy_(d["s"], non_blocking=True)
-            gx_h.copy_(d["gx"], non_blocking=True)
             g_h.copy_(d["g"], non_blocking=True)
             returned[i].record(down)
 
@@ -672,7 +668,7 @@ def time_e2e(layer, args, world, dev):
     return {"value": world * ke * w.neuron_steps / (ems / 1e3), "unit": UNIT,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": ke,
             "ms_per_step": ems / ke, "streams": 3,
-            "timing": "wall clock, host waits for each step's results",
+            "timing": "wall clock, host waits for each step's result (the parameter gradients)",
             "launch_geometry": f"the headline call (one forward and one backward of B={w.B}), "
                                "two device buffer sets alternating"}
 
