@@ -16,6 +16,8 @@ namespace dendsn {
 // Sums the block partials of every channel in a fixed order and writes the parameter
 // gradients (grad_beta only when requested). One thread per (channel, gradient slot).
 __global__ void param_grad_finalize_kernel(const FinArgs F) {
+    pdl_wait();
+    pdl_trigger();
     const Geometry &g = F.g;
     const int NP = 2 * g.K + 2 * g.Kb + 1;
     const int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -54,8 +56,21 @@ cudaError_t launch_finalize(const FinArgs &a, cudaStream_t s) {
     const int64_t n = (int64_t)a.g.C * (2 * a.g.K + 2 * a.g.Kb + 1);
     const int threads = 256;
     const int blocks = (int)((n + threads - 1) / threads);
+#if DENDSN_PDL
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)blocks);
+    cfg.blockDim = dim3((unsigned)threads);
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, param_grad_finalize_kernel, a);
+#else
     param_grad_finalize_kernel<<<blocks, threads, 0, s>>>(a);
     return cudaGetLastError();
+#endif
 }
 
 namespace {

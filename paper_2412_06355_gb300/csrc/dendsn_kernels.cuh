@@ -946,6 +946,7 @@ __device__ __forceinline__ int64_t lane_x_offset(int64_t j, int sub, int KT, int
 template <int K, int G, int PSI, typename XT, int LAYOUT>
 __global__ void __launch_bounds__(fwd_threads(K), lane_compartments(K) >= 8 ? 2 : DENDSN_FWD_MINB)
 dendsn_forward_kernel(const FwdArgs A) {
+    pdl_wait();
     constexpr int NT = fwd_threads(K);
     constexpr int KT = lane_compartments(K);
     constexpr int LPN = K / KT;
@@ -1124,6 +1125,7 @@ dendsn_forward_kernel(const FwdArgs A) {
         } else {
             rows(no{}, no{}, tc0{}, no{});
         }
+        pdl_trigger();
         cp_async_wait<0>();
         return;
     }
@@ -1207,6 +1209,7 @@ dendsn_forward_kernel(const FwdArgs A) {
 template <int K, int G, int PSI, typename XT>
 __global__ void __launch_bounds__(fwd_threads(K), K >= 8 ? 2 : DENDSN_FWD_MINB)
 dendsn_forward_staged_kernel(const FwdArgs A) {
+    pdl_wait();
     constexpr int NT = fwd_threads(K);
     constexpr int KT = K;                        // one lane per neuron
     constexpr int D = kFwdDepth;
@@ -1401,6 +1404,7 @@ template <int K, int G, int PSI, typename XT, int L, int LAYOUT, bool BETA, bool
 __global__ void __launch_bounds__(bwd_threads(bwd_lane_compartments(K, G, xt_code<XT>(), L)),
                                   bwd_threads(bwd_lane_compartments(K, G, xt_code<XT>(), L)) == 128 ? 3 : 2)
 dendsn_backward_kernel(const BwdArgs A) {
+    pdl_wait();
     constexpr int KT = bwd_lane_compartments(K, G, xt_code<XT>(), L);
     constexpr int NT = bwd_threads(KT);
     constexpr int LPN = K / KT;
@@ -1717,6 +1721,7 @@ dendsn_backward_kernel(const BwdArgs A) {
     for (int a = 0; a < NA1; ++a)
         if (!pos.active || (a < KT && P.stateless)) v[a] = 0.f;
     if constexpr (BASYNC || GSA) cp_async_wait<0>();
+    pdl_trigger();
     block_partials<KT, G, LPN, NT>(g, pos, v, reinterpret_cast<float *>(sregion), A.partials);
 }
 
@@ -1754,6 +1759,7 @@ dendsn_backward_kernel(const BwdArgs A) {
 template <int K, int PSI, typename XT, int L, bool BETA, bool GSA>
 __global__ void __launch_bounds__(bwd_threads(K), bwd_threads(K) == 128 ? DENDSN_PHASED_MINB : 2)
 dendsn_backward_phased_kernel(const BwdArgs A) {
+    pdl_wait();
     constexpr int KT = K;
     constexpr int NT = bwd_threads(KT);
     constexpr int N2 = KT / 2;
@@ -1939,6 +1945,7 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
     for (int a = 0; a < NA1; ++a)
         if (!pos.active || (a < KT && P.stateless)) v[a] = 0.f;
     cp_async_wait<0>();
+    pdl_trigger();
     block_partials<KT, 1, 1, NT>(g, pos, v, reinterpret_cast<float *>(sregion), A.partials);
 }
 
@@ -1962,6 +1969,7 @@ dendsn_backward_phased_kernel(const BwdArgs A) {
 template <int K, int PSI, int L, bool BETA>
 __global__ void __launch_bounds__(bwd_threads(K), 3)
 dendsn_backward_phased_vs_kernel(const BwdArgs A) {
+    pdl_wait();
     using XT = __nv_bfloat16;
     constexpr int KT = K;
     constexpr int NT = bwd_threads(KT);
@@ -2126,6 +2134,7 @@ dendsn_backward_phased_vs_kernel(const BwdArgs A) {
     for (int a = 0; a < NA1; ++a)
         if (!pos.active || (a < KT && P.stateless)) v[a] = 0.f;
     cp_async_wait<0>();
+    pdl_trigger();
     block_partials<KT, 1, 1, NT>(g, pos, v, reinterpret_cast<float *>(sregion), A.partials);
 }
 
@@ -2149,6 +2158,7 @@ dendsn_backward_phased_vs_kernel(const BwdArgs A) {
 template <int PSI, int LAYOUT, bool BETA>
 __global__ void __launch_bounds__(256, 2)
 dendsn_backward_rowpair_kernel(const BwdArgs A) {
+    pdl_wait();
     constexpr int K = 8, KT = 4, LPN = 2, L = 4, NT = 256;
     constexpr int NA = acc_count<KT, 1>();
     using V = XIO<float, KT, LAYOUT>;
@@ -2413,6 +2423,7 @@ dendsn_backward_rowpair_kernel(const BwdArgs A) {
     for (int i = 0; i < NA1; ++i)
         if (!pos.active || (i < KT && P.stateless)) v[i] = 0.f;
     cp_async_wait<0>();
+    pdl_trigger();
     block_partials<KT, 1, LPN, NT>(g, pos, v, reinterpret_cast<float *>(sregion), A.partials);
 }
 
@@ -2436,8 +2447,22 @@ cudaError_t launch_or_query(Kern kernel, const Args &a, int blocks, int threads,
     cudaError_t e = allow_smem(kernel, bytes);
     if (e != cudaSuccess) return e;
     if (resident) return resident_blocks(reinterpret_cast<const void *>(kernel), threads, bytes, resident);
+#if DENDSN_PDL
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)blocks);
+    cfg.blockDim = dim3((unsigned)threads);
+    cfg.dynamicSmemBytes = bytes;
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, a);
+#else
     kernel<<<blocks, threads, bytes, s>>>(a);
     return cudaGetLastError();
+#endif
 }
 
 template <int K, int G, int PSI, int XT, int LAYOUT>

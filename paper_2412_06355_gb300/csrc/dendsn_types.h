@@ -19,6 +19,27 @@ constexpr int lane_compartments(int K) { return K < 8 ? K : 8; }
 constexpr int bwd_lane_compartments(int K, int G, int xt, int L) {
     return (K >= 8 && G == 1 && xt == 0 && L <= 4) ? 4 : lane_compartments(K);
 }
+#ifdef __CUDACC__
+// Programmatic dependent launch.
+// The library's kernels are launched with programmatic stream serialization: a kernel's
+// launch overlaps the end of the one before it in the stream, and waits in pdl_wait for
+// that one's completion and memory before touching global memory (whole steps 1-2% faster
+// on the conv and token layers: the launch gaps between forward, backward and finalize).
+#ifndef DENDSN_PDL
+#define DENDSN_PDL 1
+#endif
+// Waits for the grid this one was launched after (and its memory) when launched with
+// programmatic stream serialization; a no-op otherwise. Called before any global access.
+__device__ __forceinline__ void pdl_wait() {
+    if (DENDSN_PDL) asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+// Lets the next grid in the stream begin launching once every block of this one has called
+// it or exited (that grid still waits for this one's completion in pdl_wait).
+__device__ __forceinline__ void pdl_trigger() {
+    if (DENDSN_PDL) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+#endif
+
 // Whether the backward takes the phased kernel: rows of one full chunk (T == L) of whole
 // 8-compartment neurons (one lane each), one compartment per branch, compartments
 // innermost, no residual term. The forward of such a layer keeps V^s for it when the
