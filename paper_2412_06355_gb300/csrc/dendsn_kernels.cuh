@@ -31,9 +31,11 @@
 // one full chunk of whole 8-compartment neurons take dendsn_backward_phased_kernel,
 // which runs a row in phases (recompute into shared memory, soma in registers,
 // dendritic reverse scan one compartment pair at a time) and gives bit-identical
-// results with fewer live registers. 4-step rows of 8-compartment float32 neurons on
-// two lanes take dendsn_backward_rowpair_kernel: the same phases over two rows per
-// thread, each paired instruction carrying one compartment of both rows.
+// results with fewer live registers; for bfloat16 layers whose forward kept V^s in the
+// saved buffer, dendsn_backward_phased_vs_kernel skips the recompute of the soma and
+// rescans only V^d, per compartment pair, in registers. 4-step rows of 8-compartment
+// float32 neurons on two lanes take dendsn_backward_rowpair_kernel: the same phases over
+// two rows per thread, each paired instruction carrying one compartment of both rows.
 //
 // Arithmetic. With one compartment per branch (G = 1) the per-compartment work is
 // done two compartments at a time with the paired fp32 instructions of sm_100+
@@ -42,7 +44,8 @@
 // Address arithmetic is pointer increments; 64-bit divisions happen once per thread.
 //
 // Waits. The kernels never spin: cp.async.wait_group waits on the thread's own copies,
-// __syncwarp / __syncthreads on threads that always reach them.
+// __syncwarp / __syncthreads on threads that always reach them, griddepcontrol.wait on
+// the completion of the grid launched before this one in the stream.
 #pragma once
 
 #include <cuda_bf16.h>
