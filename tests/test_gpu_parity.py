@@ -456,3 +456,44 @@ def test_concurrent_streams_match_sequential_calls():
         assert torch.equal(s0, s1)
         for key in g0:
             assert torch.equal(g0[key], g1[key]), key
+
+
+def test_chained_layers_with_torch_kernels_between_calls():
+    """The library's kernels start early behind the kernel before them in the stream and wait
+    for it before reading: two layers chained through torch kernels (layer 1's spikes mixed
+    into layer 2's input, layer 2's dL/dX reduced into layer 1's dL/dS), with no
+    synchronisation between the calls, give the bits of the same chain run with a
+    synchronisation after every operation."""
+    w1 = workloads.Workload("ch1", T=8, B=3, N=2 * 128, K=8, G=1, C=2, inner=128, dtype="bf16",
+                            psi="mh", reset="soft", seed=71)
+    w2 = workloads.Workload("ch2", T=8, B=3, N=2 * 128, K=4, G=1, C=2, inner=128, dtype="bf16",
+                            psi="mh", reset="hard", seed=72)
+    c1, c2 = binding.config_of(w1), binding.config_of(w2)
+    i1, i2 = (to_dev(workloads.make_inputs(w, "cpu")) for w in (w1, w2))
+    p1 = [i1[k] for k in ("alpha", "xi", "zeta", "kappa")]
+    p2 = [i2[k] for k in ("alpha", "xi", "zeta", "kappa")]
+    mix = torch.randn(w2.K, generator=torch.Generator().manual_seed(5)).to("cuda", torch.bfloat16)
+
+    def chain(sync):
+        step = torch.cuda.synchronize if sync else (lambda: None)
+        sv1, sc1 = binding.workspace(c1)
+        sv2, sc2 = binding.workspace(c2)
+        s1, _ = binding.forward(c1, i1["x"], *p1, None, saved=sv1)
+        step()
+        x2 = (s1.unsqueeze(-1) * mix + i2["x"]).contiguous()        # torch kernels
+        step()
+        s2, _ = binding.forward(c2, x2, *p2, None, saved=sv2)
+        step()
+        g2 = binding.backward(c2, x2, *p2, None, i2["gs"] * s2, None, sv2, sc2)
+        step()
+        gs1 = (g2["gx"].float() @ mix.float()).to(torch.bfloat16)     # torch kernels
+        step()
+        g1 = binding.backward(c1, i1["x"], *p1, None, gs1, None, sv1, sc1, want_beta=True)
+        torch.cuda.synchronize()
+        return [s1, s2] + [g2[k] for k in sorted(g2)] + [g1[k] for k in sorted(g1)]
+
+    ref = chain(True)
+    for _ in range(3):
+        got = chain(False)
+        for a, b in zip(ref, got):
+            assert torch.equal(a, b)
