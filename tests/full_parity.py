@@ -17,7 +17,9 @@ Bounds (the stated ones, no allowance):
            below what float32 evaluation of the method reaches (a plain float32 restatement,
            tests/f32_restatement.py, misses it on every large layer); the report also gives
            the worst error over the 1e-6 rms bound.
-Neurons with an ambiguous step get zero dL/dS on both sides, as in tests/parity.py.
+Neurons with an ambiguous step get zero dL/dS on both sides, as in tests/parity.py, and so
+do, for the identity branch with one compartment per branch, neurons whose u comes within
+float32 rounding of the kink of |u| at 0 (reading A22; counted in the report).
 
 V^s comes from a second forward with the V^s output (the same step function; its spikes
 must equal the production forward's bit for bit).
@@ -61,9 +63,12 @@ def _maps(w, n0, n1):
     return chan, mrow
 
 
-def run(w, threads: int | None = None, slice_steps: int = 1 << 22) -> dict:
+def run(w, threads: int | None = None, slice_steps: int = 1 << 22, want_beta: bool = False) -> dict:
     """Runs the layer on cuda:0 and compares every neuron with the oracle. Returns a report
-    (per-quantity worst error / bound and counts); raises nothing itself."""
+    (per-quantity worst error / bound and counts); raises nothing itself. want_beta: the
+    backward build with dL/dbeta (a learnable somatic decay), compared like the other
+    parameter gradients."""
+    params = PARAMS + (("gbeta",) if want_beta else ())
     assert w.layout == "kinner", "full-size parity reads x in the [T, B, N, K] layout"
     t_start = time.perf_counter()
     threads = threads or os.cpu_count() or 1
@@ -99,9 +104,31 @@ def run(w, threads: int | None = None, slice_steps: int = 1 << 22) -> dict:
         ratio = np.where(vm, np.abs(got_v - v_o) / bound, 0.0)
         sm = t_idx < first[None]
         mism = int(((got_s != s_o) & sm).sum())
-        return dict(amb=first < w.T, v_ratio=float(ratio.max()) if ratio.size else 0.0,
+        kink = _kink_ambiguous(n0, n1, x_h[:, b, n0:n1], chan, prm_h)
+        return dict(amb=(first < w.T) | kink, kink=int(kink.sum()),
+                    v_ratio=float(ratio.max()) if ratio.size else 0.0,
                     v_bad=int((ratio > 1.0).sum()), spike_mismatch=int(mism),
                     spikes=float(s_o.sum()), nonbinary=int(((got_s != 0) & (got_s != 1)).sum()))
+
+    def _kink_ambiguous(n0, n1, xs, chan, prm):
+        """Identity branch, one compartment per branch: dpsi/du = sign(u) jumps at u = 0,
+        so a neuron whose u comes within float32 rounding of 0 at some step has its sign,
+        and with it the gradient, decided by rounding (reading A22). The float64 scan of
+        Eq. methods-compartment here gives u = (V^d - xi)/zeta; the rounding scale is that
+        of the float32 evaluation u = V^d * (1/zeta) + (-xi/zeta), with V^d carrying the
+        scan's accumulated rounding (up to 1/(1 - alpha) units of 2^-24 relative)."""
+        if w.psi != "identity" or w.G != 1 or w.stateless:
+            return np.zeros(n1 - n0, dtype=bool)
+        alpha, xi, zeta = (t.double().numpy()[chan] for t in prm[:3])          # [m, K]
+        xv = xs.double().numpy()                                                 # [T, m, K]
+        vd = np.zeros_like(xv[0])
+        amb = np.zeros(n1 - n0, dtype=bool)
+        for t in range(w.T):
+            vd = alpha * vd + xv[t]
+            u = (vd - xi) / zeta
+            scale = (np.abs(vd) * (8 + 2 / (1 - alpha)) + 8 * np.abs(xi)) / zeta
+            amb |= (np.abs(u) < 2.0 ** -24 * scale).any(axis=1)
+        return amb
 
     with ThreadPoolExecutor(threads) as ex:
         r1 = list(ex.map(fwd_job, sl))
@@ -113,7 +140,7 @@ def run(w, threads: int | None = None, slice_steps: int = 1 << 22) -> dict:
     # ---- the backward on the GPU with the ambiguous neurons' upstream gradient removed
     gsp = gs.clone()
     gsp[:, amb.cuda()] = 0
-    g = binding.backward(cfg, x, *prm, mask, gsp, None, saved, scratch)
+    g = binding.backward(cfg, x, *prm, mask, gsp, None, saved, scratch, want_beta=want_beta)
     torch.cuda.synchronize()
     gx = g["gx"]
     rms_gx_gpu = float(torch.sqrt(torch.mean(gx.double() ** 2)).item()) if gx.numel() else 0.0
@@ -145,7 +172,7 @@ def run(w, threads: int | None = None, slice_steps: int = 1 << 22) -> dict:
                     ratio_bare=float(ratio_bare.max()) if ratio.size else 0.0,
                     bad_bare=int((ratio_bare > 1.0).sum()),
                     ss=float(np.sum(want * want)), worst=worst,
-                    params={k: ref[k] for k in PARAMS})
+                    params={k: ref[k] for k in params})
 
     with ThreadPoolExecutor(threads) as ex:
         r2 = list(ex.map(bwd_job, sl))
@@ -157,9 +184,11 @@ def run(w, threads: int | None = None, slice_steps: int = 1 << 22) -> dict:
     best = max(r2, key=lambda r: r["ratio_bare"])
     rep = dict(
         workload=w.name, T=w.T, B=w.B, N=w.N, K=w.K, dtype=w.dtype, psi=w.psi, reset=w.reset,
+        want_beta=want_beta,
         neurons=w.B * w.N, elements_gx=n_gx, slices=len(sl), threads=threads,
         forward_spikes_equal=same_spikes,
         ambiguous_neurons=int(amb.sum()),
+        kink_ambiguous_neurons=sum(r["kink"] for r in r1),
         spike_rate=sum(r["spikes"] for r in r1) / max(1, w.neuron_steps),
         spike_mismatches=sum(r["spike_mismatch"] for r in r1),
         nonbinary_spikes=sum(r["nonbinary"] for r in r1),
@@ -171,7 +200,7 @@ def run(w, threads: int | None = None, slice_steps: int = 1 << 22) -> dict:
         gx_elements_over_bare_bound=sum(r["bad_bare"] for r in r2), gx_worst_bare=best["worst"],
         gx_pass=max(r["excess"] for r in r2) <= atol_x,
         seconds=dict(oracle_forward=t_fwd - t_start, oracle_backward=t_bwd - t_fwd))
-    for k in PARAMS:
+    for k in params:
         want = sum(r["params"][k] for r in r2)
         got = g[k].double().cpu().numpy()
         err = np.abs(got - want)
@@ -199,7 +228,7 @@ def failures(rep: dict) -> list:
                    f"worst over the 1e-6 rms bound at {rep['gx_worst_bare']})")
     if abs(rep["gx_rms_gpu"] - rep["gx_rms_oracle"]) > 1e-4 * max(rep["gx_rms_oracle"], 1e-30):
         bad.append("grad_x RMS of GPU and oracle disagree")
-    for k in PARAMS:
+    for k in PARAMS + (("gbeta",) if rep.get("want_beta") else ()):
         if not rep[f"{k}_pass"]:
             bad.append(f"{k} out of bound (worst {rep[k + '_max_err_over_bound']:.3g} x bound)")
     return bad

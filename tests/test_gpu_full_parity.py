@@ -51,3 +51,26 @@ def test_full_layer_every_neuron(name):
     bad = full_parity.failures(rep)
     assert not bad, f"{name}: " + "; ".join(bad)
     assert rep["spike_rate"] > 0.0
+
+
+@pytest.mark.parametrize("name,kw", [("deepconv_bf16", dict(plif=True)), ("conv", dict(plif=True)),
+                                     ("deepconv_bf16", dict(psi="identity")),
+                                     ("token_dbg", dict(psi="identity"))],
+                         ids=["deepconv_bf16-plif", "conv-plif", "deepconv_bf16-identity",
+                              "token_dbg-identity"])
+def test_full_layer_variants_every_neuron(name, kw):
+    """The builds with dL/dbeta (a learnable somatic decay; compared with the oracle's
+    per-channel dL/dbeta like the other parameter gradients) and the identity branch, at full
+    size, every neuron, at the same bounds."""
+    plif = kw.pop("plif", False)
+    w = WORKLOADS[name].with_(**kw)
+    rep = full_parity.run(w, want_beta=plif)
+    out = os.environ.get("DENDSN_PARITY_REPORT")
+    if out:
+        os.makedirs(out, exist_ok=True)
+        tag = "plif" if plif else kw.get("psi", "")
+        with open(os.path.join(out, f"full_{name}_{tag}.json"), "w") as f:
+            json.dump(rep, f, indent=1)
+    bad = full_parity.failures(rep)
+    assert not bad, f"{name} {kw} plif={plif}: " + "; ".join(bad)
+
