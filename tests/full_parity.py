@@ -69,7 +69,7 @@ def run(w, threads: int | None = None, slice_steps: int = 1 << 22, want_beta: bo
     backward build with dL/dbeta (a learnable somatic decay), compared like the other
     parameter gradients."""
     params = PARAMS + (("gbeta",) if want_beta else ())
-    assert w.layout == "kinner", "full-size parity reads x in the [T, B, N, K] layout"
+    paper = w.layout == "paper"         # x and dL/dX compared in the [T, B, N, K] order
     t_start = time.perf_counter()
     threads = threads or os.cpu_count() or 1
     cfg = binding.config_of(w)
@@ -83,7 +83,7 @@ def run(w, threads: int | None = None, slice_steps: int = 1 << 22, want_beta: bo
     torch.cuda.synchronize()
     same_spikes = bool(torch.equal(s_prod, s_v))
     del s_v
-    x_h = x.cpu()
+    x_h = workloads.from_paper_layout(x.cpu(), w.N, w.K, w.inner) if paper else x.cpu()
     prm_h = [t.cpu() for t in prm]
     mask_h = None if mask is None else mask.cpu()
     ocfg = _ocfg(w)
@@ -142,7 +142,7 @@ def run(w, threads: int | None = None, slice_steps: int = 1 << 22, want_beta: bo
     gsp[:, amb.cuda()] = 0
     g = binding.backward(cfg, x, *prm, mask, gsp, None, saved, scratch, want_beta=want_beta)
     torch.cuda.synchronize()
-    gx = g["gx"]
+    gx = workloads.from_paper_layout(g["gx"], w.N, w.K, w.inner) if paper else g["gx"]
     rms_gx_gpu = float(torch.sqrt(torch.mean(gx.double() ** 2)).item()) if gx.numel() else 0.0
     gsp_h = gsp.cpu()
     rtol_x = BF16_RTOL if w.dtype == "bf16" else G_RTOL

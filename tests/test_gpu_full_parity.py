@@ -53,22 +53,28 @@ def test_full_layer_every_neuron(name):
     assert rep["spike_rate"] > 0.0
 
 
-@pytest.mark.parametrize("name,kw", [("deepconv_bf16", dict(plif=True)), ("conv", dict(plif=True)),
-                                     ("deepconv_bf16", dict(psi="identity")),
-                                     ("token_dbg", dict(psi="identity"))],
-                         ids=["deepconv_bf16-plif", "conv-plif", "deepconv_bf16-identity",
-                              "token_dbg-identity"])
+VARIANTS = [("deepconv_bf16", dict(plif=True)), ("conv", dict(plif=True)),
+            ("deepconv_bf16", dict(psi="identity")), ("token_dbg", dict(psi="identity")),
+            ("conv_paper_p4b2", dict()), ("conv", dict(stateless=True)),
+            ("conv", dict(residual=True)), ("token_dbg", dict(residual=True))]
+
+
+@pytest.mark.parametrize("name,kw", VARIANTS,
+                         ids=[n + "-" + ("-".join(f"{k}={v}" for k, v in kw.items()) or "layer")
+                              for n, kw in VARIANTS])
 def test_full_layer_variants_every_neuron(name, kw):
     """The builds with dL/dbeta (a learnable somatic decay; compared with the oracle's
-    per-channel dL/dbeta like the other parameter gradients) and the identity branch, at full
-    size, every neuron, at the same bounds."""
+    per-channel dL/dbeta like the other parameter gradients), the identity branch, the
+    paper's (C_o, P, H, W) layout with two compartments per branch, the Stateless dendrite and
+    the residual term, at full size, every neuron, at the same bounds."""
+    kw = dict(kw)
     plif = kw.pop("plif", False)
     w = WORKLOADS[name].with_(**kw)
     rep = full_parity.run(w, want_beta=plif)
     out = os.environ.get("DENDSN_PARITY_REPORT")
     if out:
         os.makedirs(out, exist_ok=True)
-        tag = "plif" if plif else kw.get("psi", "")
+        tag = "plif" if plif else "-".join(f"{k}={v}" for k, v in kw.items()) or "layer"
         with open(os.path.join(out, f"full_{name}_{tag}.json"), "w") as f:
             json.dump(rep, f, indent=1)
     bad = full_parity.failures(rep)
