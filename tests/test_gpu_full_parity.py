@@ -56,7 +56,9 @@ def test_full_layer_every_neuron(name):
 VARIANTS = [("deepconv_bf16", dict(plif=True)), ("conv", dict(plif=True)),
             ("deepconv_bf16", dict(psi="identity")), ("token_dbg", dict(psi="identity")),
             ("conv_paper_p4b2", dict()), ("conv", dict(stateless=True)),
-            ("conv", dict(residual=True)), ("token_dbg", dict(residual=True))]
+            ("conv", dict(residual=True)), ("token_dbg", dict(residual=True)),
+            ("conv", dict(mask_p=0.5)), ("conv", dict(detach_reset=True)),
+            ("deepconv_bf16", dict(reset="hard"))]
 
 
 @pytest.mark.parametrize("name,kw", VARIANTS,
@@ -65,8 +67,9 @@ VARIANTS = [("deepconv_bf16", dict(plif=True)), ("conv", dict(plif=True)),
 def test_full_layer_variants_every_neuron(name, kw):
     """The builds with dL/dbeta (a learnable somatic decay; compared with the oracle's
     per-channel dL/dbeta like the other parameter gradients), the identity branch, the
-    paper's (C_o, P, H, W) layout with two compartments per branch, the Stateless dendrite and
-    the residual term, at full size, every neuron, at the same bounds."""
+    paper's (C_o, P, H, W) layout with two compartments per branch, the Stateless dendrite,
+    the residual term, per-channel branch masks, the detached reset and the hard reset of the
+    kept-V^s backward, at full size, every neuron, at the same bounds."""
     kw = dict(kw)
     plif = kw.pop("plif", False)
     w = WORKLOADS[name].with_(**kw)
